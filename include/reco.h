@@ -1,0 +1,184 @@
+/*
+ * reco.h -- C ABI of libreco, the GB300 (sm_103a) library for the data-parallel
+ * hot path of ReCo, "Fewer Tokens, Smaller Cache: Reward-Coordinated Efficient
+ * Reasoning": reward-set retention (Eq. 1), attention-guided cache scoring
+ * (Eq. 2), per-head top-m selection with in-place compaction (Sec. 3.2), decode
+ * attention over the ragged compacted cache, the reward-banded reflection
+ * penalty (Eq. 3-4) and the answer-perplexity stop test (Eq. 5-6).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Pointers are DEVICE pointers owned by the caller unless marked "host".
+ *    The library never allocates device memory: calls that need scratch take a
+ *    caller-owned workspace sized by reco_workspace_bytes().
+ *  - Device calls are asynchronous on the given stream and return after the
+ *    launches are queued.  They return RECO_OK, or an error status before
+ *    launching anything when a host-side check fails (nothing is modified then).
+ *  - Problems only visible on the device (a length outside its range, an id or
+ *    token outside [0, V)) never make a kernel read or write out of bounds: the
+ *    affected unit is skipped and a sticky device error word is set.
+ *    reco_check() synchronises the stream, returns RECO_EDEVICE if the word is
+ *    set, and clears it.
+ *  - reco_last_error() returns the calling thread's last error message.
+ *  - Nothing throws across this ABI.
+ *
+ * Cache layout (struct reco_kv): K and V are separate contiguous arrays of shape
+ * [n_layers][B][H_kv][L_cap][d], one row of d elements per cached token, rows of
+ * one (layer, sequence, KV head) "unit" contiguous.  lens[n_layers][B][H_kv]
+ * (int32, device) holds each unit's current length; rows >= lens are unused and
+ * never read.  Query head hq belongs to KV head hq / G with G = H_q / H_kv.
+ */
+#ifndef RECO_H
+#define RECO_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RECO_OK = 0,
+    RECO_EINVAL = 1,       /* bad argument (checked on the host, before any launch) */
+    RECO_EUNSUPPORTED = 2, /* valid but not implemented (e.g. head_dim not 64 or 128) */
+    RECO_ECUDA = 3,        /* a CUDA runtime call failed */
+    RECO_EDEVICE = 4       /* the device error word was set by an earlier kernel */
+} reco_status;
+
+typedef enum { RECO_F32 = 0, RECO_BF16 = 1 } reco_dtype;
+
+typedef struct {
+    void *k;          /* device, [n_layers][B][H_kv][L_cap][d], dtype */
+    void *v;          /* device, same shape and dtype as k */
+    int n_layers;     /* >= 1 */
+    int B;            /* sequences, >= 1 */
+    int H_q;          /* query heads, a multiple of H_kv */
+    int H_kv;         /* KV heads, >= 1 */
+    int L_cap;        /* rows allocated per unit, >= 1 */
+    int d;            /* head dimension: 64 or 128 */
+    reco_dtype dtype; /* RECO_F32 or RECO_BF16 */
+} reco_kv;
+
+typedef enum { RECO_OP_SCORE = 0, RECO_OP_SELECT = 1, RECO_OP_DECODE = 2, RECO_OP_PPL = 3 } reco_op;
+
+/* ---------------------------------------------------------------- host helpers */
+
+/* Eq. 1 (Sec. 3.2): lambda_i = base - delta * (v_i - mean) / (v_max - v_min),
+ * the statistics taken over rewards[0..n-1] (host, float32, step order, the
+ * last entry being the current step's v_i).  When v_max == v_min the adjustment
+ * is 0.  Computed in double.  RECO_EINVAL if n < 1 or a pointer is NULL.       */
+reco_status reco_retention_ratio(const float *rewards, int n, double base, double delta,
+                                 double *ratio_out);
+
+/* m_i = lambda_i * L (Sec. 3.2): floor(ratio * L) clamped to [w, L].  m counts the
+ * w window tokens that are always kept.  RECO_EINVAL unless 1 <= w <= L.       */
+reco_status reco_keep_count(double ratio, int L, int w, int32_t *m_out);
+
+/* Eq. 3 band of reward v: 0 (v <= tau_l), 1 (tau_l < v < tau_h), 2 (v >= tau_h);
+ * the penalty is 0, beta/2, beta.  float32 comparisons.                       */
+int reco_penalty_band(float v, float tau_l, float tau_h);
+
+/* Sec. 3.3 early-stop probe: 1 when v_prev >= tau_h and v_cur >= tau_h.       */
+int reco_probe_trigger(float v_prev, float v_cur, float tau_h);
+
+/* Workspace bytes the device call `op` needs for this cache shape (and window w
+ * for RECO_OP_SCORE, answer batch B*n passed in `w` for RECO_OP_PPL).  The size
+ * does not depend on the device or on lens.  Alignment: 256 bytes.            */
+reco_status reco_workspace_bytes(reco_op op, const reco_kv *kv, int w, size_t *bytes_out);
+
+/* Thread-local message describing the last non-OK status ("" if none).        */
+const char *reco_last_error(void);
+
+/* Synchronise `stream`; RECO_EDEVICE (and clear) if a kernel set the device
+ * error word, RECO_ECUDA if the stream reported a CUDA error.                  */
+reco_status reco_check(cudaStream_t stream);
+
+/* ---------------------------------------------------------------- device calls */
+
+/* Eq. 2 (Sec. 3.2, attention-guided selection) for every unit of the cache.
+ * For unit (layer, b, h) of length L = lens[unit] and window w:
+ *   logit[g,t,j] = scale * q_win[layer,b,h*G+g,t,:] . K[unit, j, :]
+ *   window query t sits at position L-w+t and sees keys j <= L-w+t (causal);
+ *   raw[j]  = (1/G) * sum_g sum_t softmax_j(logit[g,t,:])
+ *   scores[unit, j] = max(raw[i] : |i-j| <= pool_kernel/2, 0 <= i < L-w)
+ * for the candidates j in [0, L-w); entries j >= L-w are left unchanged.
+ *   q_win  : [n_layers][B][H_q][w][d], same dtype as the cache (device)
+ *   lens   : [n_layers][B][H_kv] int32 (device), w <= lens <= L_cap
+ *   scores : [n_layers][B][H_kv][L_cap] float32 (device, written)
+ *   pool_kernel: odd, >= 1 (1 = Eq. 2 as printed); scale: e.g. 1/sqrt(d)
+ *   ws     : workspace of reco_workspace_bytes(RECO_OP_SCORE, kv, w) bytes
+ * A unit with lens outside [w, L_cap] is skipped (device error word set).     */
+reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, int w,
+                             int pool_kernel, float scale, float *scores, void *ws, size_t ws_bytes,
+                             cudaStream_t stream);
+
+/* Top-m selection and in-place compaction (Sec. 3.2: keep the m_i best tokens,
+ * the latest w always retained; compress the L cached tokens down to m_i).
+ * For unit (layer, b, h) with L = lens[unit] and m = keep[b]:
+ *   kept = the m-w candidates j < L-w with the largest scores[unit, j] (float32
+ *          order; equal scores keep the lower index) followed by L-w .. L-1,
+ *          in ascending order;
+ *   K[unit, r] = K[unit, kept[r]] and V[unit, r] = V[unit, kept[r]] for r < m
+ *          (in place, row order preserved); lens[unit] = m.
+ *   keep     : [B] int32 (device), w <= keep[b] <= lens (m == L is a no-op)
+ *   kept_idx : [n_layers][B][H_kv][L_cap] int32 (device) or NULL; if given, the
+ *              first m entries of each unit receive `kept`
+ *   ws       : workspace of reco_workspace_bytes(RECO_OP_SELECT, kv, w) bytes
+ * A unit with an out-of-range length or keep count is left untouched (device
+ * error word set).                                                             */
+reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t *lens,
+                                const int32_t *keep, int w, int32_t *kept_idx, void *ws,
+                                size_t ws_bytes, cudaStream_t stream);
+
+/* Decode attention over the ragged compacted cache: the per-token attention whose
+ * cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2, main results).
+ * If k_new and v_new are both non-NULL, each unit first appends its new row at
+ * index lens[unit] (which must be < L_cap) and the length grows by one; lens is
+ * updated when the kernel finishes.  Then for every query head hq of unit u:
+ *   out[layer,b,hq,:] = softmax_j(scale * q[layer,b,hq,:] . K[u,j,:]) V[u,j,:],
+ *   j over the unit's rows, lse[layer,b,hq] = natural log of the softmax sum.
+ *   q            : [n_layers][B][H_q][d], cache dtype (device)
+ *   k_new, v_new : [n_layers][B][H_kv][d], cache dtype (device) or both NULL
+ *   out          : [n_layers][B][H_q][d] of out_dtype (RECO_F32 or RECO_BF16)
+ *   lse          : [n_layers][B][H_q] float32 or NULL
+ *   ws           : workspace of reco_workspace_bytes(RECO_OP_DECODE, kv, 0) bytes
+ * A unit with a length outside [0, L_cap] (or no room to append) writes zeros
+ * and lse = -inf, and sets the device error word.                              */
+reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,
+                             int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
+                             void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* Eq. 3 + Eq. 4 (Sec. 3.3, reward-banded reflection penalty), in place:
+ *   beta_b = 0, beta/2 or beta by the band of rewards[b] (float32 compares);
+ *   logits[b, u] -= beta_b once for each distinct id u in ids[0..n_ids-1];
+ *   all other logits are left bit-for-bit unchanged.
+ *   logits  : [B][V] float32 (device, in/out)
+ *   ids     : [n_ids] int32 (device); ids outside [0, V) are skipped and set the
+ *             device error word
+ *   rewards : [B] float32 (device), the just-completed step's v_i per sequence
+ *   beta_out: [B] float32 (device) or NULL, receives beta_b                     */
+reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
+                                 const float *rewards, float tau_l, float tau_h, float beta,
+                                 float *beta_out, cudaStream_t stream);
+
+/* Eq. 5 + Eq. 6 (Sec. 3.3, early stopping via answer confidence):
+ *   lp[b,t] = logits[b,t,tokens[b,t]] - logsumexp(logits[b,t,:])   (natural log)
+ *   ppl[b]  = exp(-(1/n_b) sum_{t < n_b} lp[b,t]),  stop[b] = ppl[b] <= tau_p
+ * with n_b = n_valid[b] (clamped to n) or n when n_valid is NULL; n_b == 0 gives
+ * ppl = NaN and stop = 0.  Raw logits, no penalty, temperature 1.
+ *   logits : [B][n][V] float32 (device); tokens : [B][n] int32 (device)
+ *   ppl    : [B] float32 (device, written); stop : [B] uint8 (device, written)
+ *   ws     : workspace of reco_workspace_bytes(RECO_OP_PPL, NULL, B*n) bytes
+ * A token outside [0, V) makes that sequence's ppl NaN and stop 0 and sets the
+ * device error word.                                                           */
+reco_status reco_answer_ppl(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B,
+                            int n, int V, float tau_p, float *ppl, uint8_t *stop, void *ws,
+                            size_t ws_bytes, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RECO_H */

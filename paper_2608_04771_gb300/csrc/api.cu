@@ -1,0 +1,285 @@
+// api.cu -- the extern "C" entry points of libreco (declared in include/reco.h):
+// host-side argument checks, workspace carving, the sticky device error word, and
+// the host helpers for Eq. 1, the keep count, the Eq. 3 band and the probe trigger.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <mutex>
+#include <string>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+reco_status fail(reco_status st, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+reco_status cuda_fail(cudaError_t e, const char *where)
+{
+    return fail(RECO_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+// One sticky error word per device; kernels receive its device address.
+__device__ unsigned int g_reco_error_word;
+
+std::mutex g_mu;
+unsigned *g_err_addr[128];
+int g_sm_count[128];
+
+reco_status error_word(unsigned **out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 128) return fail(RECO_EUNSUPPORTED, "device index %d out of range", dev);
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_err_addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_reco_error_word);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(error word)");
+        g_err_addr[dev] = (unsigned *)p;
+    }
+    *out = g_err_addr[dev];
+    return RECO_OK;
+}
+
+bool al16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+reco_status check_kv(const reco_kv *kv, bool need_kv_ptrs = true)
+{
+    if (!kv) return fail(RECO_EINVAL, "kv descriptor is NULL");
+    if (kv->n_layers < 1 || kv->B < 1 || kv->H_kv < 1 || kv->H_q < 1 || kv->L_cap < 1)
+        return fail(RECO_EINVAL, "kv dimensions must be >= 1 (layers %d, B %d, H_q %d, H_kv %d, L_cap %d)",
+                    kv->n_layers, kv->B, kv->H_q, kv->H_kv, kv->L_cap);
+    if (kv->H_q % kv->H_kv != 0) return fail(RECO_EINVAL, "H_q (%d) is not a multiple of H_kv (%d)", kv->H_q, kv->H_kv);
+    if (kv->dtype != RECO_F32 && kv->dtype != RECO_BF16) return fail(RECO_EINVAL, "unknown dtype %d", (int)kv->dtype);
+    if (kv->d != 64 && kv->d != 128) return fail(RECO_EUNSUPPORTED, "head dim %d (supported: 64, 128)", kv->d);
+    long long units = (long long)kv->n_layers * kv->B * kv->H_kv;
+    if (units > 65535) return fail(RECO_EUNSUPPORTED, "%lld units exceed 65535", units);
+    if (need_kv_ptrs) {
+        if (!kv->k || !kv->v) return fail(RECO_EINVAL, "K or V pointer is NULL");
+        if (!al16(kv->k) || !al16(kv->v)) return fail(RECO_EINVAL, "K and V must be 16-byte aligned");
+    }
+    return RECO_OK;
+}
+
+reco_status check_ws(void *ws, size_t have, size_t need)
+{
+    if (need == 0) return RECO_OK;
+    if (!ws) return fail(RECO_EINVAL, "workspace is NULL (%zu bytes needed)", need);
+    if (((uintptr_t)ws & 255u) != 0) return fail(RECO_EINVAL, "workspace must be 256-byte aligned");
+    if (have < need) return fail(RECO_EINVAL, "workspace has %zu bytes, %zu needed", have, need);
+    return RECO_OK;
+}
+
+}  // namespace
+
+namespace reco {
+bool score_shape_supported(const reco_kv &kv, int w);
+
+int device_sm_count()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return 148;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_sm_count[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 148;
+        g_sm_count[dev] = n;
+    }
+    return g_sm_count[dev];
+}
+}  // namespace reco
+
+extern "C" {
+
+const char *reco_last_error(void) { return g_last_error.c_str(); }
+
+reco_status reco_retention_ratio(const float *rewards, int n, double base, double delta, double *ratio_out)
+{
+    if (!rewards || !ratio_out) return fail(RECO_EINVAL, "NULL pointer");
+    if (n < 1) return fail(RECO_EINVAL, "reward history is empty");
+    double sum = 0.0, vmin = rewards[0], vmax = rewards[0];
+    for (int i = 0; i < n; ++i) {
+        const double v = rewards[i];
+        sum += v;
+        vmin = v < vmin ? v : vmin;
+        vmax = v > vmax ? v : vmax;
+    }
+    const double mean = sum / (double)n, range = vmax - vmin;
+    *ratio_out = range == 0.0 ? base : base - delta * (((double)rewards[n - 1] - mean) / range);
+    return RECO_OK;
+}
+
+reco_status reco_keep_count(double ratio, int L, int w, int32_t *m_out)
+{
+    if (!m_out) return fail(RECO_EINVAL, "NULL pointer");
+    if (w < 1 || L < w) return fail(RECO_EINVAL, "need 1 <= w <= L (w %d, L %d)", w, L);
+    if (!(ratio == ratio)) return fail(RECO_EINVAL, "ratio is NaN");
+    const double f = floor(ratio * (double)L);
+    *m_out = f < (double)w ? w : (f > (double)L ? L : (int32_t)f);
+    return RECO_OK;
+}
+
+int reco_penalty_band(float v, float tau_l, float tau_h)
+{
+    if (v <= tau_l) return 0;
+    if (v >= tau_h) return 2;
+    return 1;
+}
+
+int reco_probe_trigger(float v_prev, float v_cur, float tau_h) { return v_prev >= tau_h && v_cur >= tau_h; }
+
+reco_status reco_workspace_bytes(reco_op op, const reco_kv *kv, int w, size_t *bytes_out)
+{
+    if (!bytes_out) return fail(RECO_EINVAL, "NULL pointer");
+    reco_status st;
+    switch (op) {
+    case RECO_OP_SCORE:
+        if ((st = check_kv(kv, false)) != RECO_OK) return st;
+        if (w < 1) return fail(RECO_EINVAL, "window w must be >= 1");
+        *bytes_out = reco::score_ws_layout(*kv, w, nullptr).bytes;
+        return RECO_OK;
+    case RECO_OP_SELECT:
+        if ((st = check_kv(kv, false)) != RECO_OK) return st;
+        *bytes_out = reco::select_ws_layout(*kv, nullptr).bytes;
+        return RECO_OK;
+    case RECO_OP_DECODE:
+        if ((st = check_kv(kv, false)) != RECO_OK) return st;
+        *bytes_out = reco::decode_ws_layout(*kv, nullptr).bytes;
+        return RECO_OK;
+    case RECO_OP_PPL:
+        if (w < 0) return fail(RECO_EINVAL, "answer rows B*n must be >= 0");
+        *bytes_out = reco::align256((size_t)w * 4);
+        return RECO_OK;
+    }
+    return fail(RECO_EINVAL, "unknown op %d", (int)op);
+}
+
+reco_status reco_check(cudaStream_t stream)
+{
+    cudaError_t e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    unsigned *p;
+    reco_status st = error_word(&p);
+    if (st != RECO_OK) return st;
+    unsigned h = 0;
+    if ((e = cudaMemcpyAsync(&h, p, sizeof h, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+        return cuda_fail(e, "read error word");
+    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    if (h) {
+        if ((e = cudaMemsetAsync(p, 0, sizeof h, stream)) != cudaSuccess) return cuda_fail(e, "clear error word");
+        if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+        return fail(RECO_EDEVICE, "device error word 0x%x:%s%s%s%s%s%s", h, (h & reco::ERR_LEN) ? " length-out-of-range" : "",
+                    (h & reco::ERR_KEEP) ? " keep-out-of-range" : "", (h & reco::ERR_ID) ? " id-out-of-range" : "",
+                    (h & reco::ERR_TOKEN) ? " token-out-of-range" : "", (h & reco::ERR_ROOM) ? " no-room-to-append" : "",
+                    (h & reco::ERR_INTERNAL) ? " internal-check" : "");
+    }
+    return RECO_OK;
+}
+
+reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, int w, int pool_kernel,
+                             float scale, float *scores, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    reco_status st = check_kv(kv);
+    if (st != RECO_OK) return st;
+    if (!q_win || !lens || !scores) return fail(RECO_EINVAL, "NULL q_win, lens or scores");
+    if (!al16(q_win) || ((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u))
+        return fail(RECO_EINVAL, "q_win must be 16-byte aligned, lens and scores 4-byte aligned");
+    if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
+    if (pool_kernel < 1 || (pool_kernel & 1) == 0) return fail(RECO_EINVAL, "pool_kernel %d must be odd and >= 1", pool_kernel);
+    if (!(scale == scale)) return fail(RECO_EINVAL, "scale is NaN");
+    const int G = kv->H_q / kv->H_kv;
+    if ((long long)G * w > 4096) return fail(RECO_EUNSUPPORTED, "G*w = %lld window rows exceed 4096", (long long)G * w);
+    if (!reco::score_shape_supported(*kv, w))
+        return fail(RECO_EUNSUPPORTED, "G*w*d too large for the scoring kernels (G %d, w %d, d %d)", G, w, kv->d);
+    reco::ScoreWs lay = reco::score_ws_layout(*kv, w, ws);
+    if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_score(*kv, q_win, lens, w, pool_kernel, scale, scores, lay, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_score_cache launch");
+}
+
+reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t *lens, const int32_t *keep, int w,
+                                int32_t *kept_idx, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    reco_status st = check_kv(kv);
+    if (st != RECO_OK) return st;
+    if (!scores || !lens || !keep) return fail(RECO_EINVAL, "NULL scores, lens or keep");
+    if (((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u) || ((uintptr_t)keep & 3u) || ((uintptr_t)kept_idx & 3u))
+        return fail(RECO_EINVAL, "scores, lens, keep and kept_idx must be 4-byte aligned");
+    if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
+    reco::SelectWs lay = reco::select_ws_layout(*kv, ws);
+    if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_select_compact(*kv, scores, lens, keep, w, kept_idx, lay, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_select_compact launch");
+}
+
+reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new, const void *v_new, int32_t *lens,
+                             float scale, void *out, reco_dtype out_dtype, float *lse, void *ws, size_t ws_bytes,
+                             cudaStream_t stream)
+{
+    reco_status st = check_kv(kv);
+    if (st != RECO_OK) return st;
+    if (!q || !lens || !out) return fail(RECO_EINVAL, "NULL q, lens or out");
+    if ((k_new == nullptr) != (v_new == nullptr)) return fail(RECO_EINVAL, "k_new and v_new must both be given or both NULL");
+    if (!al16(q) || !al16(out) || (k_new && (!al16(k_new) || !al16(v_new))))
+        return fail(RECO_EINVAL, "q, out, k_new and v_new must be 16-byte aligned");
+    if (((uintptr_t)lens & 3u) || ((uintptr_t)lse & 3u)) return fail(RECO_EINVAL, "lens and lse must be 4-byte aligned");
+    if (out_dtype != RECO_F32 && out_dtype != RECO_BF16) return fail(RECO_EINVAL, "unknown out_dtype %d", (int)out_dtype);
+    const int G = kv->H_q / kv->H_kv;
+    if (G > 16) return fail(RECO_EUNSUPPORTED, "G = %d query heads per KV head (at most 16)", G);
+    if (!(scale == scale)) return fail(RECO_EINVAL, "scale is NaN");
+    reco::DecodeWs lay = reco::decode_ws_layout(*kv, ws);
+    if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_decode(*kv, q, k_new, v_new, lens, scale, out, out_dtype, lse, lay, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_decode_attn launch");
+}
+
+reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
+                                 float tau_l, float tau_h, float beta, float *beta_out, cudaStream_t stream)
+{
+    if (B < 1 || V < 1 || n_ids < 0) return fail(RECO_EINVAL, "need B >= 1, V >= 1, n_ids >= 0");
+    if (!logits || !rewards || (n_ids > 0 && !ids)) return fail(RECO_EINVAL, "NULL logits, rewards or ids");
+    if (B > 65535) return fail(RECO_EUNSUPPORTED, "B = %d exceeds 65535", B);
+    if (!(beta >= 0.f)) return fail(RECO_EINVAL, "beta must be >= 0");
+    unsigned *err;
+    reco_status st = error_word(&err);
+    if (st != RECO_OK) return st;
+    cudaError_t e = reco::launch_penalty(logits, B, V, ids, n_ids, rewards, tau_l, tau_h, beta, beta_out, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_reflect_penalty launch");
+}
+
+reco_status reco_answer_ppl(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B, int n, int V,
+                            float tau_p, float *ppl, uint8_t *stop, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    if (B < 1 || n < 0 || V < 1) return fail(RECO_EINVAL, "need B >= 1, n >= 0, V >= 1");
+    if (B > 65535 || n > 65535) return fail(RECO_EUNSUPPORTED, "B or n exceeds 65535");
+    if (!ppl || !stop || (n > 0 && (!logits || !tokens))) return fail(RECO_EINVAL, "NULL logits, tokens, ppl or stop");
+    if (((uintptr_t)logits & 3u)) return fail(RECO_EINVAL, "logits must be 4-byte aligned");
+    reco_status st = check_ws(ws, ws_bytes, reco::align256((size_t)B * n * 4));
+    if (st != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_ppl(logits, tokens, n_valid, B, n, V, tau_p, ppl, stop, (float *)ws, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_answer_ppl launch");
+}
+
+}  // extern "C"

@@ -1,0 +1,62 @@
+// internal.h -- launcher interface between the C ABI layer (api.cu) and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/reco.h"
+
+namespace reco {
+
+// Keys per scoring work item (one CTA per (unit, chunk) in both scoring passes).
+constexpr int kScoreChunk = 2048;
+// Upper bound on decode split-K work items beyond one per unit.
+constexpr int kDecodeMaxTarget = 8192;
+
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct ScoreWs {  // float regions carved from the caller's workspace
+    float *part_m, *part_z;  // [units][n_chunks][R]  per-chunk row max (log2) / row sum
+    float *rowb;             // [units][R]            log2 of the row normaliser
+    float *raw;              // [units][L_cap]        unpooled scores
+    size_t bytes;
+};
+
+struct SelectWs {
+    int32_t *idx;    // [units][L_cap] kept indices (when the caller passes none)
+    int32_t *count;  // [units] rows to compact (0 = skip unit)
+    size_t bytes;
+};
+
+struct DecodeWs {
+    int32_t *counters;  // [2 + units]: work counter, finished warps, per-unit tickets
+    float *part_ml;     // [max_items][G][2]  (m log2, l)
+    float *part_o;      // [max_items][G][d]  unnormalised output
+    int max_items;
+    size_t bytes;
+};
+
+ScoreWs score_ws_layout(const reco_kv &kv, int w, void *base);
+SelectWs select_ws_layout(const reco_kv &kv, void *base);
+DecodeWs decode_ws_layout(const reco_kv &kv, void *base);
+
+// Launchers return cudaSuccess or the launch error.  All arguments validated by the caller.
+cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, int pool,
+                         float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s);
+cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
+                                  const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
+                                  unsigned *err, cudaStream_t s);
+cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
+                          int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
+                          const DecodeWs &ws, unsigned *err, cudaStream_t s);
+cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
+                           const float *rewards, float tau_l, float tau_h, float beta, float *beta_out,
+                           unsigned *err, cudaStream_t s);
+cudaError_t launch_ppl(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B, int n,
+                       int V, float tau_p, float *ppl, uint8_t *stop, float *lp_ws, unsigned *err,
+                       cudaStream_t s);
+
+// Device properties cached per device.
+int device_sm_count();
+
+}  // namespace reco

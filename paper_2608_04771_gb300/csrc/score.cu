@@ -1,0 +1,266 @@
+// score.cu -- Eq. 2 (Sec. 3.2, attention-guided selection): per-KV-head cache scores.
+//
+// s_j = (1/G) sum_g sum_t softmax_j(scale * q_{g,t} . k_j), window query t at position
+// L-w+t seeing keys j <= L-w+t, then a max-pool over the candidate range [0, L-w).
+//
+// A softmax row needs its max and normaliser over ALL keys before any column can be
+// summed, so the scores take two passes over K:
+//   pass 1  per (unit, key chunk): per-row running max / sum in the log2 domain
+//   combine per (unit, row): merge the chunk partials -> b_r = m_r + log2 Z_r
+//   pass 2  per (unit, key chunk): column sums  sum_r 2^(c*l_rj - b_r) / G
+//   pool    per (unit, key): max over the clipped window
+// This file holds the SIMT version used for float32 caches (and any shape the
+// tensor-core version does not cover); score_tc.cu holds the bf16 tensor-core passes.
+#include "common.cuh"
+#include "internal.h"
+
+namespace reco {
+
+ScoreWs score_ws_layout(const reco_kv &kv, int w, void *base)
+{
+    size_t units = (size_t)kv.n_layers * kv.B * kv.H_kv;
+    size_t R = (size_t)(kv.H_q / kv.H_kv) * w;
+    size_t nch = ((size_t)kv.L_cap + kScoreChunk - 1) / kScoreChunk;
+    char *p = (char *)base;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        char *r = p ? p + off : nullptr;
+        off += align256(bytes);
+        return r;
+    };
+    ScoreWs ws;
+    ws.part_m = (float *)take(units * nch * R * 4);
+    ws.part_z = (float *)take(units * nch * R * 4);
+    ws.rowb = (float *)take(units * R * 4);
+    ws.raw = (float *)take(units * (size_t)kv.L_cap * 4);
+    ws.bytes = off;
+    return ws;
+}
+
+// Pass 1: one thread per window row, its query held in registers; K streamed
+// through shared memory 64 rows at a time.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) score_rowstats_simt(
+    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, int w,
+    int G, int Hq, int Hkv, int L_cap, int R, int n_chunks, float c2, float *__restrict__ part_m,
+    float *__restrict__ part_z, unsigned *err)
+{
+    constexpr int KT = 64;
+    __shared__ __align__(16) float Ks[KT][D];
+    const int chunk = blockIdx.x;
+    const long u = blockIdx.y;
+    const int r = blockIdx.z * blockDim.x + threadIdx.x;
+    const int L = lens[u];
+    if (L < w || L > L_cap) {
+        if (chunk == 0 && blockIdx.z == 0 && threadIdx.x == 0) raise_error(err, ERR_LEN);
+        return;
+    }
+    const int j0 = chunk * kScoreChunk;
+    const int j1 = min(j0 + kScoreChunk, L);
+    const long lb = u / Hkv;
+    const int h = (int)(u % Hkv);
+    const bool row_ok = r < R;
+    const int g = row_ok ? r / w : 0, t = row_ok ? r % w : 0;
+    const int jmax = L - w + t;
+    float q[D];
+    {
+        const T *qp = q_win + (((lb * Hq) + (long)h * G + g) * w + t) * D;
+#pragma unroll
+        for (int c = 0; c < D; ++c) q[c] = row_ok ? to_float(qp[c]) : 0.f;
+    }
+    float m = -INFINITY, z = 0.f;
+    const T *Kp = K + u * (long)L_cap * D;
+    for (int jt = j0; jt < j1; jt += KT) {
+        const int nk = min(KT, j1 - jt);
+        __syncthreads();
+        for (int e = threadIdx.x; e < KT * D; e += blockDim.x) {
+            int jj = e / D, c = e % D;
+            Ks[jj][c] = jj < nk ? to_float(Kp[(long)(jt + jj) * D + c]) : 0.f;
+        }
+        __syncthreads();
+        if (row_ok) {
+            for (int jj = 0; jj < nk; ++jj) {
+                if (jt + jj > jmax) break;
+                float s = 0.f;
+#pragma unroll
+                for (int c = 0; c < D; c += 4) {
+                    float4 kv = *reinterpret_cast<const float4 *>(&Ks[jj][c]);
+                    s = fmaf(q[c], kv.x, s);
+                    s = fmaf(q[c + 1], kv.y, s);
+                    s = fmaf(q[c + 2], kv.z, s);
+                    s = fmaf(q[c + 3], kv.w, s);
+                }
+                s *= c2;
+                if (s > m) {
+                    z = z * fast_exp2(m - s) + 1.f;
+                    m = s;
+                } else {
+                    z += fast_exp2(s - m);
+                }
+            }
+        }
+    }
+    if (row_ok) {
+        size_t o = ((size_t)u * n_chunks + chunk) * R + r;
+        part_m[o] = m;
+        part_z[o] = z;
+    }
+}
+
+// Merge the chunk partials of each row into b_r = m_r + log2(Z_r).
+__global__ void score_combine(const int32_t *__restrict__ lens, int w, int L_cap, int R, int n_chunks,
+                              const float *__restrict__ part_m, const float *__restrict__ part_z,
+                              float *__restrict__ rowb, long units)
+{
+    long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= units * R) return;
+    long u = i / R;
+    int r = (int)(i % R);
+    int L = lens[u];
+    if (L < w || L > L_cap) return;
+    int used = (L + kScoreChunk - 1) / kScoreChunk;
+    float m = -INFINITY, z = 0.f;
+    for (int c = 0; c < used; ++c) {
+        size_t o = ((size_t)u * n_chunks + c) * R + r;
+        lse_merge(m, z, part_m[o], part_z[o]);
+    }
+    rowb[i] = m + log2f(z);
+}
+
+// Pass 2: one thread per candidate key, its key row held in registers; the window
+// queries sit in shared memory and are read by broadcast.
+template <typename T, int D>
+__global__ void __launch_bounds__(128) score_colsum_simt(
+    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, int w,
+    int G, int Hq, int Hkv, int L_cap, int R, float c2, const float *__restrict__ rowb,
+    float *__restrict__ raw)
+{
+    extern __shared__ __align__(16) float smem[];
+    float *Qs = smem;         // [R][D]
+    float *Bs = smem + R * D; // [R]
+    const int chunk = blockIdx.x;
+    const long u = blockIdx.y;
+    const int L = lens[u];
+    if (L < w || L > L_cap) return;
+    const int nc = L - w;
+    const int j0 = chunk * kScoreChunk;
+    const int j1 = min(j0 + kScoreChunk, nc);
+    if (j0 >= j1) return;
+    const long lb = u / Hkv;
+    const int h = (int)(u % Hkv);
+    for (int e = threadIdx.x; e < R * D; e += blockDim.x) {
+        int rr = e / D, c = e % D;
+        int g = rr / w, t = rr % w;
+        Qs[e] = to_float(q_win[(((lb * Hq) + (long)h * G + g) * w + t) * D + c]);
+    }
+    for (int rr = threadIdx.x; rr < R; rr += blockDim.x) Bs[rr] = rowb[u * R + rr];
+    __syncthreads();
+    const T *Kp = K + u * (long)L_cap * D;
+    const float invG = 1.f / (float)G;
+    for (int j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
+        float k[D];
+#pragma unroll
+        for (int c = 0; c < D; ++c) k[c] = to_float(Kp[(long)j * D + c]);
+        float acc = 0.f;
+        for (int rr = 0; rr < R; ++rr) {
+            const float *qr = Qs + rr * D;
+            float s = 0.f;
+#pragma unroll
+            for (int c = 0; c < D; c += 4) {
+                float4 qv = *reinterpret_cast<const float4 *>(qr + c);
+                s = fmaf(qv.x, k[c], s);
+                s = fmaf(qv.y, k[c + 1], s);
+                s = fmaf(qv.z, k[c + 2], s);
+                s = fmaf(qv.w, k[c + 3], s);
+            }
+            acc += fast_exp2(fmaf(s, c2, -Bs[rr]));
+        }
+        raw[u * L_cap + j] = acc * invG;
+    }
+}
+
+// Max-pool over the clipped window [j - pool/2, j + pool/2] within [0, L-w).
+__global__ void score_pool(const float *__restrict__ raw, const int32_t *__restrict__ lens, int w,
+                           int L_cap, int pool, float *__restrict__ scores)
+{
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    const long u = blockIdx.y;
+    const int L = lens[u];
+    if (L < w || L > L_cap) return;
+    const int nc = L - w;
+    if (j >= nc) return;
+    const int half = pool / 2;
+    const int lo = max(0, j - half), hi = min(nc - 1, j + half);
+    const float *rp = raw + u * L_cap;
+    float m = rp[lo];
+    for (int i = lo + 1; i <= hi; ++i) m = fmaxf(m, rp[i]);
+    scores[u * L_cap + j] = m;
+}
+
+cudaError_t launch_score_tc(const reco_kv &kv, const void *q_win, const int32_t *lens, int w,
+                            float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+
+template <typename T, int D>
+static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *lens, int w, float c2,
+                              const ScoreWs &ws, unsigned *err, cudaStream_t s)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const int G = kv.H_q / kv.H_kv, R = G * w;
+    const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
+    const T *K = (const T *)kv.k;
+    int bx = R < 256 ? ((R + 31) / 32) * 32 : 256;
+    dim3 g1(nch, (unsigned)units, (R + bx - 1) / bx);
+    score_rowstats_simt<T, D><<<g1, bx, 0, s>>>(q_win, K, lens, w, G, kv.H_q, kv.H_kv, kv.L_cap, R, nch,
+                                                c2, ws.part_m, ws.part_z, err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    long n = units * R;
+    score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, w, kv.L_cap, R, nch, ws.part_m,
+                                                              ws.part_z, ws.rowb, units);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    size_t smem = ((size_t)R * D + R) * sizeof(float);
+    e = cudaFuncSetAttribute(score_colsum_simt<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    score_colsum_simt<T, D><<<dim3(nch, (unsigned)units), 128, smem, s>>>(
+        q_win, K, lens, w, G, kv.H_q, kv.H_kv, kv.L_cap, R, c2, ws.rowb, ws.raw);
+    return cudaGetLastError();
+}
+
+// Largest R*D the SIMT pass 2 keeps in shared memory.
+constexpr size_t kSimtMaxQ = 200 * 1024 / 4;
+
+bool score_shape_supported(const reco_kv &kv, int w)
+{
+    size_t R = (size_t)(kv.H_q / kv.H_kv) * w;
+    return (kv.d == 64 || kv.d == 128) && (R * kv.d + R) <= kSimtMaxQ;
+}
+
+cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, int pool,
+                         float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s)
+{
+    const float c2 = scale * kLog2e;
+    cudaError_t e = cudaSuccess;
+    bool used_tc = false;
+    if (kv.dtype == RECO_BF16) {
+        e = launch_score_tc(kv, q_win, lens, w, c2, ws, err, s, &used_tc);
+        if (e != cudaSuccess) return e;
+    }
+    if (!used_tc) {
+        if (kv.dtype == RECO_F32)
+            e = kv.d == 64 ? score_simt<float, 64>(kv, (const float *)q_win, lens, w, c2, ws, err, s)
+                           : score_simt<float, 128>(kv, (const float *)q_win, lens, w, c2, ws, err, s);
+        else
+            e = kv.d == 64
+                    ? score_simt<__nv_bfloat16, 64>(kv, (const __nv_bfloat16 *)q_win, lens, w, c2, ws, err, s)
+                    : score_simt<__nv_bfloat16, 128>(kv, (const __nv_bfloat16 *)q_win, lens, w, c2, ws, err,
+                                                     s);
+        if (e != cudaSuccess) return e;
+    }
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, w, kv.L_cap,
+                                                                            pool, scores);
+    return cudaGetLastError();
+}
+
+}  // namespace reco

@@ -1,0 +1,232 @@
+// select.cu -- top-m selection and in-place compaction (Sec. 3.2: keep the m_i
+// highest-scoring tokens with the latest w always retained, then compress the L
+// cached tokens down to m_i).
+//
+// select_topm: one CTA per (layer, sequence, KV head).  A 4 x 8-bit radix select
+// over order-preserving uint32 keys of the float32 scores finds the (m-w)-th
+// largest key T and how many keys equal to T are still needed; one ordered pass
+// then emits every candidate with key > T plus the first `need` with key == T in
+// index order.  The result is sorted and ties go to the lower index, with no sort.
+//
+// compact_rows: one CTA per (unit, K|V, 128-byte column slice).  kept[] is strictly
+// increasing, so kept[r] >= r: the source of destination r is never a row that an
+// earlier destination overwrote.  Each CTA walks its destinations in order, reads a
+// chunk of source rows, synchronises, then writes the chunk; reads of later chunks
+// may run ahead of earlier writes because their sources lie above every row written
+// so far.  Rows with kept[r] == r are not moved.
+#include "common.cuh"
+#include "internal.h"
+
+namespace reco {
+
+SelectWs select_ws_layout(const reco_kv &kv, void *base)
+{
+    size_t units = (size_t)kv.n_layers * kv.B * kv.H_kv;
+    char *p = (char *)base;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        char *r = p ? p + off : nullptr;
+        off += align256(bytes);
+        return r;
+    };
+    SelectWs ws;
+    ws.idx = (int32_t *)take(units * (size_t)kv.L_cap * 4);
+    ws.count = (int32_t *)take(units * 4);
+    ws.bytes = off;
+    return ws;
+}
+
+__device__ __forceinline__ uint32_t order_key(float f)
+{
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Exclusive block scan of a 0/1 flag.  `tot` must hold NT/32 + 1 ints.
+template <int NT>
+__device__ __forceinline__ int block_scan_flag(bool flag, int *tot, int &total)
+{
+    const unsigned lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const unsigned bal = __ballot_sync(0xffffffffu, flag);
+    const int in_warp = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) tot[wid] = __popc(bal);
+    __syncthreads();
+    if (wid == 0) {
+        int v = lane < NT / 32 ? tot[lane] : 0;
+        int incl = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            int n = __shfl_up_sync(0xffffffffu, incl, o);
+            if ((int)lane >= o) incl += n;
+        }
+        if (lane < NT / 32) tot[lane] = incl - v;
+        if (lane == 31) tot[NT / 32] = incl;
+    }
+    __syncthreads();
+    const int res = tot[wid] + in_warp;
+    total = tot[NT / 32];
+    __syncthreads();
+    return res;
+}
+
+template <int NT>
+__global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scores, int32_t *lens,
+                                                  const int32_t *__restrict__ keep, int w, int B, int Hkv,
+                                                  int L_cap, int32_t *__restrict__ idx_out,
+                                                  int32_t *__restrict__ count, unsigned *err)
+{
+    __shared__ int hist[256];
+    __shared__ int tot[NT / 32 + 1];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_remaining;
+    const long u = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int b = (int)((u / Hkv) % B);
+    const int L = lens[u], m = keep[b];
+    if (L < w || L > L_cap || m < w || m > L) {
+        if (tid == 0) {
+            count[u] = 0;
+            raise_error(err, (L < w || L > L_cap) ? ERR_LEN : ERR_KEEP);
+        }
+        return;
+    }
+    const int nc = L - w, kc = m - w;
+    const float *s = scores + u * L_cap;
+    int32_t *idx = idx_out + u * L_cap;
+    if (kc == nc) {  // keep everything: identity, nothing moves
+        for (int j = tid; j < L; j += NT) idx[j] = j;
+        if (tid == 0) count[u] = m;
+        return;
+    }
+    uint32_t T = 0xffffffffu;
+    int need = 0;
+    if (kc > 0) {
+        if (tid == 0) {
+            s_prefix = 0;
+            s_remaining = kc;
+        }
+        uint32_t mask = 0;
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            for (int i = tid; i < 256; i += NT) hist[i] = 0;
+            __syncthreads();
+            const uint32_t prefix = s_prefix;
+            const int remaining = s_remaining;
+            for (int jb = 0; jb < nc; jb += NT) {
+                const int j = jb + tid;
+                const bool valid = j < nc;
+                const uint32_t key = valid ? order_key(s[j]) : 0u;
+                const bool match = valid && (key & mask) == prefix;
+                const uint32_t bin = (key >> shift) & 255u;
+                const unsigned peers = __match_any_sync(0xffffffffu, match ? bin : 256u + lane);
+                if (match && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+            }
+            __syncthreads();
+            if (tid < 32) {  // find the bin holding the remaining-th largest key
+                int c8[8], sum = 0;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    c8[i] = hist[255 - 8 * lane - i];
+                    sum += c8[i];
+                }
+                int incl = sum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    int n = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += n;
+                }
+                int cum = incl - sum;
+                if (cum < remaining && remaining <= incl) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        if (cum + c8[i] >= remaining) {
+                            s_prefix = prefix | ((uint32_t)(255 - 8 * lane - i) << shift);
+                            s_remaining = remaining - cum;
+                            break;
+                        }
+                        cum += c8[i];
+                    }
+                }
+            }
+            mask |= 255u << shift;
+            __syncthreads();
+        }
+        T = s_prefix;
+        need = s_remaining;
+    }
+    int base_pos = 0, base_eq = 0;
+    for (int jb = 0; jb < nc; jb += NT) {
+        const int j = jb + tid;
+        const bool valid = j < nc;
+        const uint32_t key = valid ? order_key(s[j]) : 0u;
+        const bool gt = valid && key > T;
+        const bool eq = valid && key == T;
+        int eq_tot, f_tot;
+        const int eq_rank = block_scan_flag<NT>(eq, tot, eq_tot) + base_eq;
+        const bool flag = gt || (eq && eq_rank < need);
+        const int pos = block_scan_flag<NT>(flag, tot, f_tot) + base_pos;
+        if (flag) idx[pos] = j;
+        base_eq += eq_tot;
+        base_pos += f_tot;
+    }
+    for (int t = tid; t < w; t += NT) idx[kc + t] = nc + t;
+    if (tid == 0) {
+        count[u] = m;
+        lens[u] = m;
+    }
+}
+
+__global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int32_t *__restrict__ idx_all,
+                                                    const int32_t *__restrict__ count, int L_cap,
+                                                    int row_bytes, unsigned *err)
+{
+    constexpr int P = 8;  // 16-byte pieces per 128-byte slice
+    constexpr int U = 4;  // rows per thread in flight
+    const long u = blockIdx.x;
+    const int m = count[u];
+    if (m == 0) return;
+    char *base = (blockIdx.y == 0 ? K : V) + u * (long)L_cap * row_bytes;
+    const int32_t *idx = idx_all + u * L_cap;
+    const int rows_per_pass = blockDim.x / P;
+    const int my_row = threadIdx.x / P;
+    const int off = blockIdx.z * 128 + (threadIdx.x % P) * 16;
+    for (int r0 = 0; r0 < m; r0 += U * rows_per_pass) {
+        uint4 v[U];
+        int dst[U];
+#pragma unroll
+        for (int i = 0; i < U; ++i) {
+            const int r = r0 + i * rows_per_pass + my_row;
+            dst[i] = -1;
+            if (r < m) {
+                const int src = idx[r];
+                if (src < r || src >= L_cap) {  // never trust an index outside [r, L_cap)
+                    raise_error(err, ERR_INTERNAL);
+                } else if (src != r) {
+                    v[i] = *reinterpret_cast<const uint4 *>(base + (long)src * row_bytes + off);
+                    dst[i] = r;
+                }
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < U; ++i)
+            if (dst[i] >= 0) *reinterpret_cast<uint4 *>(base + (long)dst[i] * row_bytes + off) = v[i];
+    }
+}
+
+cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
+                                  const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
+                                  unsigned *err, cudaStream_t s)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    int32_t *idx = kept_idx ? kept_idx : ws.idx;
+    select_topm<1024><<<(unsigned)units, 1024, 0, s>>>(scores, lens, keep, w, kv.B, kv.H_kv, kv.L_cap,
+                                                       idx, ws.count, err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int row_bytes = kv.d * (kv.dtype == RECO_F32 ? 4 : 2);
+    dim3 grid((unsigned)units, 2, row_bytes / 128);
+    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, idx, ws.count, kv.L_cap, row_bytes, err);
+    return cudaGetLastError();
+}
+
+}  // namespace reco

@@ -1,0 +1,177 @@
+"""Thin ctypes binding over libreco.so, with the C ABI's names (include/reco.h).
+
+Only argument marshalling happens here: torch tensors supply device pointers and
+the current CUDA stream; every step of the hot path runs in the library's kernels.
+There is no fallback: if the library is missing or a call fails, this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+import torch
+
+_LIB_PATH = Path(__file__).resolve().parent / "_build" / "libreco.so"
+_lib = None
+
+RECO_OK, RECO_EINVAL, RECO_EUNSUPPORTED, RECO_ECUDA, RECO_EDEVICE = range(5)
+RECO_F32, RECO_BF16 = 0, 1
+RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL = range(4)
+
+EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
+           "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
+           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_answer_ppl")
+
+
+class RecoError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"reco status {status}: {msg}")
+        self.status = status
+
+
+class reco_kv(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("n_layers", ctypes.c_int),
+                ("B", ctypes.c_int), ("H_q", ctypes.c_int), ("H_kv", ctypes.c_int),
+                ("L_cap", ctypes.c_int), ("d", ctypes.c_int), ("dtype", ctypes.c_int)]
+
+
+def library_path() -> Path:
+    return _LIB_PATH
+
+
+def lib():
+    """Load libreco.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not _LIB_PATH.exists():
+        raise RuntimeError(f"{_LIB_PATH} is missing: build it with __graft_entry__.build() "
+                           "or `python -m paper_2608_04771_gb300.build`")
+    L = ctypes.CDLL(str(_LIB_PATH))
+    vp, i32, f32, f64, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_double, ctypes.c_size_t
+    kvp = ctypes.POINTER(reco_kv)
+    L.reco_retention_ratio.argtypes = [vp, i32, f64, f64, ctypes.POINTER(f64)]
+    L.reco_keep_count.argtypes = [f64, i32, i32, ctypes.POINTER(ctypes.c_int32)]
+    L.reco_penalty_band.argtypes = [f32, f32, f32]
+    L.reco_penalty_band.restype = i32
+    L.reco_probe_trigger.argtypes = [f32, f32, f32]
+    L.reco_probe_trigger.restype = i32
+    L.reco_workspace_bytes.argtypes = [i32, kvp, i32, ctypes.POINTER(sz)]
+    L.reco_last_error.argtypes = []
+    L.reco_last_error.restype = ctypes.c_char_p
+    L.reco_check.argtypes = [vp]
+    L.reco_score_cache.argtypes = [kvp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
+    L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
+    L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
+    L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
+    L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
+    for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
+                 "reco_score_cache", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty",
+                 "reco_answer_ppl"):
+        getattr(L, name).restype = i32
+    _lib = L
+    return L
+
+
+def _ok(status: int):
+    if status != RECO_OK:
+        raise RecoError(status, lib().reco_last_error().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dtype_code(dt):
+    if dt == torch.float32:
+        return RECO_F32
+    if dt == torch.bfloat16:
+        return RECO_BF16
+    raise TypeError(f"unsupported dtype {dt}")
+
+
+def make_kv(K: torch.Tensor, V: torch.Tensor, H_q: int) -> reco_kv:
+    """Describe contiguous [layers, B, H_kv, L_cap, d] K and V tensors."""
+    if K.shape != V.shape or K.dtype != V.dtype or K.dim() != 5:
+        raise ValueError("K and V must be [layers, B, H_kv, L_cap, d] with equal shape and dtype")
+    if not (K.is_contiguous() and V.is_contiguous()):
+        raise ValueError("K and V must be contiguous")
+    Ly, B, Hkv, Lcap, d = K.shape
+    return reco_kv(K.data_ptr(), V.data_ptr(), Ly, B, H_q, Hkv, Lcap, d, _dtype_code(K.dtype))
+
+
+# ---------------------------------------------------------------- host helpers
+def reco_retention_ratio(rewards, base: float = 0.25, delta: float = 0.1) -> float:
+    import numpy as np
+    r = np.ascontiguousarray(rewards, dtype=np.float32).ravel()
+    out = ctypes.c_double()
+    _ok(lib().reco_retention_ratio(r.ctypes.data, int(r.size), float(base), float(delta), ctypes.byref(out)))
+    return out.value
+
+
+def reco_keep_count(ratio: float, L: int, w: int) -> int:
+    out = ctypes.c_int32()
+    _ok(lib().reco_keep_count(float(ratio), int(L), int(w), ctypes.byref(out)))
+    return out.value
+
+
+def reco_penalty_band(v: float, tau_l: float = 0.4, tau_h: float = 0.8) -> int:
+    return lib().reco_penalty_band(v, tau_l, tau_h)
+
+
+def reco_probe_trigger(v_prev: float, v_cur: float, tau_h: float = 0.8) -> bool:
+    return bool(lib().reco_probe_trigger(v_prev, v_cur, tau_h))
+
+
+def reco_workspace_bytes(op: int, kv: reco_kv | None, w: int = 0) -> int:
+    out = ctypes.c_size_t()
+    _ok(lib().reco_workspace_bytes(op, ctypes.byref(kv) if kv is not None else None, int(w),
+                                   ctypes.byref(out)))
+    return out.value
+
+
+def workspace(op: int, kv: reco_kv | None, w: int = 0, device="cuda") -> torch.Tensor:
+    n = reco_workspace_bytes(op, kv, w)
+    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+
+
+def reco_check(stream=None):
+    _ok(lib().reco_check(_stream(stream)))
+
+
+# ---------------------------------------------------------------- device calls
+def reco_score_cache(kv: reco_kv, q_win, lens, w: int, pool_kernel: int, scale: float, scores, ws,
+                     stream=None):
+    _ok(lib().reco_score_cache(ctypes.byref(kv), _ptr(q_win), _ptr(lens), int(w), int(pool_kernel),
+                               float(scale), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_select_compact(kv: reco_kv, scores, lens, keep, w: int, kept_idx, ws, stream=None):
+    _ok(lib().reco_select_compact(ctypes.byref(kv), _ptr(scores), _ptr(lens), _ptr(keep), int(w),
+                                  _ptr(kept_idx), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_decode_attn(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, lse, ws, stream=None):
+    _ok(lib().reco_decode_attn(ctypes.byref(kv), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(lens),
+                               float(scale), _ptr(out), _dtype_code(out.dtype), _ptr(lse), _ptr(ws),
+                               ws.numel(), _stream(stream)))
+
+
+def reco_reflect_penalty(logits, ids, rewards, tau_l=0.4, tau_h=0.8, beta=4.0, beta_out=None,
+                         stream=None):
+    B, V = logits.shape
+    _ok(lib().reco_reflect_penalty(_ptr(logits), B, V, _ptr(ids), ids.numel(), _ptr(rewards),
+                                   float(tau_l), float(tau_h), float(beta), _ptr(beta_out),
+                                   _stream(stream)))
+
+
+def reco_answer_ppl(logits, tokens, n_valid, tau_p, ppl, stop, ws, stream=None):
+    B, n, V = logits.shape
+    _ok(lib().reco_answer_ppl(_ptr(logits), _ptr(tokens), _ptr(n_valid), B, n, V, float(tau_p),
+                              _ptr(ppl), _ptr(stop), _ptr(ws), ws.numel(), _stream(stream)))

@@ -130,21 +130,27 @@ def outlier_channels(wl: Workload) -> np.ndarray:
     return out
 
 
-def make_cache(wl: Workload, device="cpu", canary: bool = True):
-    """K, V of shape [layers, batch, h_kv, L_cap, d]; rows >= L are NaN when ``canary``."""
+def _cache_tensor(wl: Workload, stream: int, device, canary: bool) -> torch.Tensor:
     shape = (wl.layers, wl.batch, wl.h_kv, wl.L_cap, wl.d)
-    K = randn(shape, wl, 1, device, torch.float32)
-    V = randn(shape, wl, 2, device, torch.float32)
+    x = randn(shape, wl, stream, device, torch.float32)
     if wl.outliers:
         ch = torch.from_numpy(outlier_channels(wl)).to(device)
         for l in range(wl.layers):
             for h in range(wl.h_kv):
-                K[l, :, h, :, ch[l, h]] *= 20.0
-                V[l, :, h, :, ch[l, h]] *= 20.0
+                x[l, :, h, :, ch[l, h]] *= 20.0
     if canary and wl.L_cap > wl.L:
-        K[:, :, :, wl.L:, :] = float("nan")
-        V[:, :, :, wl.L:, :] = float("nan")
-    return K.to(wl.torch_dtype), V.to(wl.torch_dtype)
+        x[:, :, :, wl.L:, :] = float("nan")
+    y = x.to(wl.torch_dtype)
+    del x
+    return y
+
+
+def make_cache(wl: Workload, device="cpu", canary: bool = True):
+    """K, V of shape [layers, batch, h_kv, L_cap, d]; rows >= L are NaN when ``canary``.
+    The outlier channels (if any) are scaled by 20 in both K and V."""
+    K = _cache_tensor(wl, 1, device, canary)
+    V = _cache_tensor(wl, 2, device, canary)
+    return K, V
 
 
 def make_lens(wl: Workload, device="cpu") -> torch.Tensor:

@@ -1,0 +1,124 @@
+"""The C-ABI library on the CPU: it builds, loads, exports every symbol include/reco.h
+declares, its host helpers agree with the oracle, and host-side argument checks
+reject bad calls before any launch (no GPU needed, no compute calls)."""
+import ctypes
+import json
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_04771_gb300 import build as B
+from paper_2608_04771_gb300 import reco
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    B.build()
+    return reco.lib()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "reco.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*(reco_[a-z_0-9]+)\s*\(", text, flags=re.M)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    names = declared_functions()
+    assert len(names) >= 12
+    assert set(names) == set(reco.EXPORTS)
+    for n in names:
+        assert hasattr(L, n), n
+    out = os.popen(f"nm -D --defined-only {B.LIB}").read()
+    for n in names:
+        assert re.search(rf"\bT {n}\b", out), n
+
+
+def test_retention_ratio_and_keep_count_match_oracle(L):
+    g = json.load(open(os.path.join(ROOT, "tests", "golden", "eq1_retention.json")))
+    for c in g["cases"]:
+        r = reco.reco_retention_ratio(c["history"], c["base"], c["delta"])
+        assert r == oracle.retention_ratio(c["history"], c["base"], c["delta"])
+        assert reco.reco_keep_count(r, c["L"], c["w"]) == c["m"]
+    rng = np.random.default_rng(0)
+    for _ in range(2000):
+        h = rng.random(int(rng.integers(1, 30))).astype(np.float32)
+        base, delta = float(rng.uniform(0.1, 0.6)), float(rng.uniform(0, 0.35))
+        r = reco.reco_retention_ratio(h, base, delta)
+        assert r == oracle.retention_ratio(h, base, delta)  # bit-exact (same definition, same order)
+        Lc = int(rng.integers(1, 40000))
+        w = int(rng.integers(1, Lc + 1))
+        assert reco.reco_keep_count(r, Lc, w) == oracle.keep_count(r, Lc, w)
+
+
+def test_band_and_trigger_match_oracle(L):
+    g = json.load(open(os.path.join(ROOT, "tests", "golden", "eq34_penalty.json")))
+    for c in g["bands"]:
+        assert reco.reco_penalty_band(c["v"], g["tau_l"], g["tau_h"]) == c["band"]
+    for c in g["probe_trigger"]:
+        assert reco.reco_probe_trigger(c["v_prev"], c["v_cur"], 0.8) == c["fire"]
+    for v in np.linspace(0, 1, 1001, dtype=np.float32):
+        assert reco.reco_penalty_band(float(v)) == oracle.penalty_band(float(v))
+
+
+def test_host_helpers_reject_bad_input(L):
+    with pytest.raises(reco.RecoError) as e:
+        reco.reco_retention_ratio([], 0.25, 0.1)
+    assert e.value.status == reco.RECO_EINVAL
+    with pytest.raises(reco.RecoError):
+        reco.reco_keep_count(0.25, 10, 11)  # w > L
+    with pytest.raises(reco.RecoError):
+        reco.reco_keep_count(0.25, 10, 0)
+
+
+def _kv(**kw):
+    d = dict(k=16, v=32, n_layers=2, B=3, H_q=8, H_kv=2, L_cap=100, d=128, dtype=reco.RECO_BF16)
+    d.update(kw)
+    return reco.reco_kv(d["k"], d["v"], d["n_layers"], d["B"], d["H_q"], d["H_kv"], d["L_cap"], d["d"],
+                        d["dtype"])
+
+
+def test_workspace_sizes(L):
+    kv = _kv()
+    s = reco.reco_workspace_bytes(reco.RECO_OP_SCORE, kv, 16)
+    units, R = 2 * 3 * 2, 4 * 16
+    assert s >= units * 100 * 4 + units * R * 4
+    assert reco.reco_workspace_bytes(reco.RECO_OP_SELECT, kv) >= units * 100 * 4
+    assert reco.reco_workspace_bytes(reco.RECO_OP_DECODE, kv) > 0
+    assert reco.reco_workspace_bytes(reco.RECO_OP_PPL, None, 64) == 256
+    with pytest.raises(reco.RecoError):
+        reco.reco_workspace_bytes(reco.RECO_OP_SCORE, _kv(d=96), 16)
+    with pytest.raises(reco.RecoError):
+        reco.reco_workspace_bytes(reco.RECO_OP_SCORE, _kv(H_q=7), 16)
+
+
+def test_device_calls_validate_before_launch(L):
+    """Bad shapes, NULLs, misalignment and short workspaces fail with EINVAL/EUNSUPPORTED
+    on the host; no kernel is launched (this machine has no GPU)."""
+    kv = _kv()
+    vp = ctypes.c_void_p
+    ws = vp(256 * 1000)
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 0, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 16, 4, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"pool_kernel" in L.reco_last_error()
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    st = L.reco_score_cache(ctypes.byref(_kv(k=17)), vp(16), vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    st = L.reco_select_compact(ctypes.byref(kv), None, vp(16), vp(16), 16, None, ws, 10, None)
+    assert st == reco.RECO_EINVAL
+    st = L.reco_decode_attn(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 0.1, vp(16), 0, None, ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"k_new" in L.reco_last_error()
+    st = L.reco_decode_attn(ctypes.byref(_kv(H_q=34, H_kv=2)), vp(16), None, None, vp(16), 0.1, vp(16), 0,
+                            None, ws, 10, None)
+    assert st == reco.RECO_EUNSUPPORTED
+    st = L.reco_reflect_penalty(vp(16), 0, 10, vp(16), 1, vp(16), 0.4, 0.8, 4.0, None, None)
+    assert st == reco.RECO_EINVAL
+    st = L.reco_answer_ppl(vp(16), vp(16), None, 2, 4, 10, 1.1, vp(16), vp(16), None, 0, None)
+    assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()

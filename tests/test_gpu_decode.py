@@ -1,0 +1,116 @@
+"""reco_decode_attn vs the oracle's softmax attention (float64), element by element,
+over ragged per-unit lengths, with and without the fused append."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import DECODE_ATOL, gpu_decode, np32
+from paper_2608_04771_gb300 import reco
+from paper_2608_04771_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2608_04771_gb300 import build
+    build.build()
+    reco.lib()
+
+
+def _oracle_decode(wl, K_np, V_np, lens_np, q_np, kn_np=None, vn_np=None):
+    K_np, V_np, lens_np = K_np.copy(), V_np.copy(), lens_np.copy()
+    if kn_np is not None:
+        for l in range(wl.layers):
+            for b in range(wl.batch):
+                for h in range(wl.h_kv):
+                    L = lens_np[l, b, h]
+                    K_np[l, b, h, L] = kn_np[l, b, h]
+                    V_np[l, b, h, L] = vn_np[l, b, h]
+                    lens_np[l, b, h] = L + 1
+    out, lse = oracle.decode_batch(q_np, np.nan_to_num(K_np), np.nan_to_num(V_np), lens_np, wl.scale())
+    return out, lse, K_np, V_np, lens_np
+
+
+def _check(wl, lens_np, append: bool, out_dtype=torch.float32, steps=1):
+    K, V = W.make_cache(wl, DEV, canary=True)
+    lens = torch.from_numpy(lens_np).to(DEV)
+    for l in range(wl.layers):
+        for b in range(wl.batch):
+            for h in range(wl.h_kv):
+                K[l, b, h, int(lens_np[l, b, h]):] = float("nan")
+                V[l, b, h, int(lens_np[l, b, h]):] = float("nan")
+    K_np, V_np, L_np = np32(K), np32(V), lens_np.copy()
+    atol = DECODE_ATOL[wl.dtype]
+    for s in range(steps):
+        q, kn, vn = W.make_decode_step(wl, s, DEV)
+        out, lse = gpu_decode(wl, K, V, lens, q, kn if append else None, vn if append else None, out_dtype)
+        reco.reco_check()
+        o_ref, lse_ref, K_np, V_np, L_np = _oracle_decode(wl, K_np, V_np, L_np, np32(q),
+                                                          np32(kn) if append else None,
+                                                          np32(vn) if append else None)
+        got = out.float().cpu().numpy()
+        tol = atol + (np.abs(o_ref) * 2.0 ** -8 if out_dtype == torch.bfloat16 else 0.0)
+        err = np.abs(got - o_ref)
+        assert (err <= tol).all(), f"step {s}: worst {err.max():.3e}"
+        lse_got = lse.cpu().numpy()
+        fin = np.isfinite(lse_ref)
+        assert np.array_equal(np.isfinite(lse_got), fin)
+        assert np.abs(lse_got[fin] - lse_ref[fin]).max(initial=0) < 1e-3
+        np.testing.assert_array_equal(lens.cpu().numpy(), L_np)
+        if append:  # the new rows landed in the cache
+            np.testing.assert_array_equal(np.nan_to_num(np32(K)), np.nan_to_num(K_np))
+            np.testing.assert_array_equal(np.nan_to_num(np32(V)), np.nan_to_num(V_np))
+
+
+@pytest.mark.parametrize("name", ["1.5b", "7b", "32b"])
+@pytest.mark.parametrize("append", [False, True])
+def test_bf16_decode_ragged(name, append):
+    base = W.WORKLOADS[name]
+    wl = base.reduced(layers=2, batch=2, L=3000, decode_steps=3)
+    rng = np.random.default_rng(7)
+    hi = wl.L_cap - (3 if append else 0)
+    lens = rng.integers(1, hi + 1, (2, 2, wl.h_kv)).astype(np.int32)
+    lens[0, 0, 0] = hi
+    lens[1, 1, 0] = 1
+    _check(wl, lens, append, steps=3 if append else 1)
+
+
+def test_bf16_decode_bf16_output_and_d64():
+    wl = W.WORKLOADS["7b"].reduced(layers=1, batch=3, L=900, decode_steps=2)
+    _check(wl, np.array([[[900, 1, 17, 899]] * 3], np.int32).reshape(1, 3, 4), True, torch.bfloat16, steps=2)
+    wl64 = W.WORKLOADS["7b"].reduced(layers=1, batch=2, h_q=8, h_kv=2, d=64, L=500, decode_steps=1)
+    _check(wl64, np.array([[[500, 37], [3, 250]]], np.int32), True)
+
+
+def test_fp32_decode_tiny_and_d128():
+    wl = W.WORKLOADS["tiny"]
+    _check(wl, np.array([[[128, 256]]], np.int32), True)
+    wl2 = W.WORKLOADS["tiny"].reduced(d=128, h_q=6, h_kv=2, L=300, decode_steps=2, batch=2)
+    _check(wl2, np.array([[[300, 5], [1, 150]]], np.int32), True, steps=2)
+
+
+def test_long_single_unit_many_splits():
+    wl = W.WORKLOADS["7b"].reduced(layers=1, batch=1, h_q=7, h_kv=1, L=40000, decode_steps=1)
+    _check(wl, np.array([[[40000]]], np.int32), True)
+
+
+def test_empty_unit_and_no_room():
+    wl = W.WORKLOADS["7b"].reduced(layers=1, batch=2, h_q=7, h_kv=1, L=64, decode_steps=0)
+    K, V = W.make_cache(wl, DEV, canary=False)
+    q, _, _ = W.make_decode_step(wl, 0, DEV)
+    lens = torch.tensor([[[0], [10]]], dtype=torch.int32, device=DEV)
+    out, lse = gpu_decode(wl, K, V, lens, q)
+    reco.reco_check()
+    assert torch.all(out[0, 0] == 0) and torch.all(torch.isneginf(lse[0, 0]))
+    # a full unit cannot take an appended row: error word, zero output, length unchanged
+    _, kn, vn = W.make_decode_step(wl.reduced(decode_steps=1), 0, DEV)
+    lens = torch.tensor([[[64], [10]]], dtype=torch.int32, device=DEV)
+    out, lse = gpu_decode(wl, K, V, lens, q, kn, vn)
+    with pytest.raises(reco.RecoError) as e:
+        reco.reco_check()
+    assert e.value.status == reco.RECO_EDEVICE
+    assert torch.all(out[0, 0] == 0) and int(lens[0, 0, 0]) == 64 and int(lens[0, 1, 0]) == 11
+    reco.reco_check()

@@ -1,0 +1,76 @@
+"""Full-size workloads in the launch configuration bench.py times (driver.HotPath),
+checked on sampled units that the oracle computes one by one."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import (DECODE_ATOL, PPL_RTOL, assert_kept_match, assert_scores_close, np32)
+from paper_2608_04771_gb300 import driver, reco
+from paper_2608_04771_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2608_04771_gb300 import build
+    build.build()
+    reco.lib()
+
+
+@pytest.mark.parametrize("name", ["7b", "1.5b", "32b"])
+def test_full_size_sampled_units(name):
+    wl = W.WORKLOADS[name]
+    hp = driver.HotPath(wl, DEV, out_dtype=torch.float32, keep_pristine=False)
+    units = [(0, 0, 0), (wl.layers // 2, wl.batch // 2, wl.h_kv - 1), (wl.layers - 1, wl.batch - 1, wl.h_kv // 2)]
+    G = wl.G
+    saved = {}
+    for (l, b, h) in units:
+        saved[(l, b, h)] = (np32(hp.K[l, b, h, :wl.L]), np32(hp.V[l, b, h, :wl.L]),
+                            np32(hp.q_win[l, b, h * G:(h + 1) * G]))
+    z0 = hp.logits.cpu().numpy().copy() if hp.has_vocab else None
+    hp.step()
+    reco.reco_check()
+    torch.cuda.synchronize()
+    check_steps = sorted({0, wl.decode_steps // 2, wl.decode_steps - 1})
+    for (l, b, h) in units:
+        K0, V0, q = saved[(l, b, h)]
+        m = int(hp.keep_host[b])
+        _, pooled = oracle.score_unit(q, K0, wl.w, wl.scale(), wl.pool)
+        got_s = hp.scores[l, b, h, :wl.L - wl.w].cpu().numpy()
+        assert_scores_close(got_s, pooled, f"{name} unit {(l, b, h)}")
+        ora_idx = oracle.select_unit(pooled.astype(np.float32), wl.L, wl.w, m)
+        gk = hp.kept[l, b, h].cpu().numpy()
+        nd = assert_kept_match(gk, ora_idx, pooled, wl.L, wl.w, m, f"{name} unit {(l, b, h)}")
+        if nd:
+            continue
+        Kc = np.zeros((wl.L_cap, wl.d), np.float32)
+        Vc = np.zeros((wl.L_cap, wl.d), np.float32)
+        Kc[:m], Vc[:m] = oracle.gather_unit(K0, ora_idx), oracle.gather_unit(V0, ora_idx)
+        dk = np32(hp.dk[:, l, b, h])
+        dv = np32(hp.dv[:, l, b, h])
+        Kc[m:m + wl.decode_steps], Vc[m:m + wl.decode_steps] = dk, dv
+        np.testing.assert_array_equal(np32(hp.K[l, b, h, :m + wl.decode_steps]), Kc[:m + wl.decode_steps])
+        np.testing.assert_array_equal(np32(hp.V[l, b, h, :m + wl.decode_steps]), Vc[:m + wl.decode_steps])
+        assert int(hp.lens[l, b, h]) == m + wl.decode_steps
+        for s in check_steps:
+            qs = np32(hp.dq[s, l, b, h * G:(h + 1) * G])
+            got = hp.out[s, l, b, h * G:(h + 1) * G].float().cpu().numpy()
+            for g in range(G):
+                o, lse = oracle.decode_unit(qs[g], Kc, Vc, m + s + 1, wl.scale())
+                assert np.abs(got[g] - o).max() <= DECODE_ATOL[wl.dtype], (name, s, l, b, h, g)
+                assert abs(float(hp.lse[s, l, b, h * G + g]) - lse) < 1e-3
+    if hp.has_vocab:
+        # the penalty ran once per decode step on the same logits buffer
+        ids = W.make_reflection_ids(wl)
+        ref = z0
+        for _ in range(wl.decode_steps):
+            ref, beta_ref, _ = oracle.reflect_penalty(ref, ids, hp.hist[:, -1], wl.tau_l, wl.tau_h, wl.beta)
+        np.testing.assert_array_equal(hp.logits.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+        np.testing.assert_array_equal(hp.beta.cpu().numpy(), beta_ref)
+        ppl_ref, stop_ref = oracle.answer_ppl(np32(hp.ans_logits), hp.ans_tokens.cpu().numpy(), None, wl.tau_p)
+        got = hp.ppl.cpu().numpy().astype(np.float64)
+        assert np.all(np.abs(got - ppl_ref) <= PPL_RTOL * ppl_ref)
+        assert np.array_equal(hp.stop.cpu().numpy().astype(bool), stop_ref)
