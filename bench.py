@@ -434,9 +434,16 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-units", type=int, default=32, help="oracle sample: units of layer 0")
     ap.add_argument("--ref-dec-steps", type=int, default=8, help="oracle sample: decode steps")
+    ap.add_argument("--layers", type=int, help="override the layer count (profiling a smaller case)")
+    ap.add_argument("--batch", type=int, help="override the batch (profiling a smaller case)")
+    ap.add_argument("--decode-steps", type=int, help="override the decode steps (profiling a smaller case)")
     args = ap.parse_args()
     from paper_2608_04771_gb300 import workloads as W
     wl = W.WORKLOADS[args.workload]
+    over = {k: v for k, v in (("layers", args.layers), ("batch", args.batch),
+                               ("decode_steps", args.decode_steps)) if v is not None}
+    if over:
+        wl = wl.reduced(**over)
     if args.impl == "reference":
         run_reference(args, wl)
     else:

@@ -185,6 +185,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// (a, b) -> bf16x2 hi = round(a, b) and lo = round((a, b) - hi).
+__device__ __forceinline__ void split_bf16(float a, float b, uint32_t &hi, uint32_t &lo)
+{
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    const float2 f = __bfloat1622float2(h);
+    hi = *reinterpret_cast<uint32_t *>(&h);
+    lo = pack_bf16(a - f.x, b - f.y);
+}
+
 __device__ __forceinline__ uint32_t word(const uint4 &v, int x)
 {
     return x == 0 ? v.x : (x == 1 ? v.y : (x == 2 ? v.z : v.w));
@@ -414,7 +423,11 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
                 o[t][2] *= a0;
                 o[t][3] *= a1;
             }
-            const uint32_t pb0 = pack_bf16(p0, p1), pb1 = pack_bf16(p2, p3);
+            // P enters the PV product as bf16 hi + lo parts (two MMAs), which keeps about
+            // 16 significant bits of each probability instead of 8.
+            uint32_t ph0, ph1, pl0, pl1;
+            split_bf16(p0, p1, ph0, pl0);
+            split_bf16(p2, p3, ph1, pl1);
 #pragma unroll
             for (int i = 0; i < NVI; ++i) {
                 const uint4 v0 = lds_u4(st + (2 * NKI + 0 * NVI + i) * 512);
@@ -424,8 +437,10 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
 #pragma unroll
                 for (int x = 0; x < 4; ++x) {
                     const uint32_t W0 = word(v0, x), W1 = word(v1, x), W2 = word(v2, x), W3 = word(v3, x);
-                    mma_bf16(o[4 * i + x], __byte_perm(W0, W1, 0x5410), __byte_perm(W0, W1, 0x7632),
-                             __byte_perm(W2, W3, 0x5410), __byte_perm(W2, W3, 0x7632), pb0, pb1);
+                    const uint32_t A0 = __byte_perm(W0, W1, 0x5410), A1 = __byte_perm(W0, W1, 0x7632);
+                    const uint32_t A2 = __byte_perm(W2, W3, 0x5410), A3 = __byte_perm(W2, W3, 0x7632);
+                    mma_bf16(o[4 * i + x], A0, A1, A2, A3, ph0, ph1);
+                    mma_bf16(o[4 * i + x], A0, A1, A2, A3, pl0, pl1);
                 }
             }
         }

@@ -35,7 +35,7 @@ def _oracle_decode(wl, K_np, V_np, lens_np, q_np, kn_np=None, vn_np=None):
 
 
 def _check(wl, lens_np, append: bool, out_dtype=torch.float32, steps=1):
-    K, V = W.make_cache(wl, DEV, canary=True)
+    K, V = W.make_cache(wl, DEV, canary=False)  # the test poisons rows >= its own lengths
     lens = torch.from_numpy(lens_np).to(DEV)
     for l in range(wl.layers):
         for b in range(wl.batch):
@@ -54,7 +54,7 @@ def _check(wl, lens_np, append: bool, out_dtype=torch.float32, steps=1):
         got = out.float().cpu().numpy()
         tol = atol + (np.abs(o_ref) * 2.0 ** -8 if out_dtype == torch.bfloat16 else 0.0)
         err = np.abs(got - o_ref)
-        assert (err <= tol).all(), f"step {s}: worst {err.max():.3e}"
+        assert (err <= tol).all(), f"step {s}: worst {np.nanmax(err):.3e}, NaN {np.isnan(err).sum()}"
         lse_got = lse.cpu().numpy()
         fin = np.isfinite(lse_ref)
         assert np.array_equal(np.isfinite(lse_got), fin)

@@ -23,7 +23,7 @@ def _lib():
 
 
 def _check(wl, lens_np, pool):
-    K, V = W.make_cache(wl, DEV, canary=True)
+    K, V = W.make_cache(wl, DEV, canary=False)  # the test poisons rows >= its own lengths
     q = W.make_qwin(wl, DEV)
     lens = torch.from_numpy(lens_np).to(DEV)
     # rows in [lens, L) are valid data the kernel must not read: poison them too
