@@ -1,23 +1,25 @@
 // decode.cu -- decode attention over the ragged compacted cache, the per-token
 // attention whose cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2).
 //
-// bf16 path (decode_mma): a persistent split-K flash-decode.  Every CTA first builds
-// the same work plan from lens: a key-chunk length C chosen so the total number of
-// (unit, chunk) items is a few per warp, and the prefix sum of chunks per unit.  Each
-// warp then takes items from an atomic counter.  An item's keys stream from HBM in
-// 16-key blocks through a private 3-stage shared-memory ring filled with cp.async
-// (zero-fill past the end); each thread copies exactly the 16-byte pieces it later
-// reads, so no barrier is needed and the piece-major layout has no bank conflicts.
-// QK^T and PV run on mma.sync m16n8k16 (bf16 in, fp32 accumulate) with the G <= 8
-// query heads of the KV head packed into one MMA tile.  The head dimension is
-// permuted consistently on the Q and K sides (and on the V and output sides) so
-// that each thread's fragments are contiguous 16-byte pieces of a row.  A unit split over several items writes partial
+// bf16 path (decode_tma): a persistent split-K flash-decode, one CTA of 8 warps per
+// SM.  Every CTA first builds the same work plan from lens: a key-chunk length C
+// chosen so the total number of (unit, chunk) items is several per warp, and the
+// prefix sum of chunks per unit.  Each warp then takes items from an atomic counter.
+// An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
+// (128-byte swizzled 16 x 64 tiles of K and V) into the warp's 3-stage ring and the
+// warp waits on the stage's mbarrier (bounded).  QK^T and PV run on mma.sync
+// m16n8k16 (bf16 in, fp32 accumulate) with the G <= 8 query heads of the KV head
+// packed into one MMA tile.  The head dimension is permuted consistently on the Q
+// and K sides (and on the V and output sides) so that each thread's fragments are
+// whole 16-byte chunks, and the swizzle makes every fragment read conflict-free.  A unit split over several items writes partial
 // (max, sum, output) triples; the last item to finish (atomic ticket, no waiting)
 // merges them.  The appended token (k_new, v_new) is read from the inputs and written
 // into the cache by the warp that covers its index; the last warp of the grid to
 // finish advances lens.
 //
 // float32 path (decode_simt): one CTA per unit, four warps over the keys, G <= 16.
+#include <cuda.h>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -199,46 +201,6 @@ __device__ __forceinline__ uint32_t word(const uint4 &v, int x)
     return x == 0 ? v.x : (x == 1 ? v.y : (x == 2 ? v.z : v.w));
 }
 
-// cp.async of one 16-byte piece into shared memory; src_bytes 0 writes zeros.
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes)
-{
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;"); }
-template <int N> __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N)); }
-
-// Issue the 16-byte pieces one thread needs for the 16-key block at kb into its slots
-// of a ring stage.  Piece p of lane l sits at ((p * 32) + l) * 16 bytes, so each warp-
-// wide shared load of piece p reads 512 contiguous bytes.  Pieces 0 .. 2*NKI-1 hold K
-// rows kb+g and kb+8+g (head-dim elements 8c + 32i ..), pieces 2*NKI .. hold V rows
-// kb+2c, kb+2c+1, kb+2c+8, kb+2c+9 (elements 8g + 64i ..).  Rows at or past k1 are
-// zero-filled; the appended row (index Lapp) comes from k_new / v_new.
-template <int D>
-__device__ __forceinline__ void issue_block(uint32_t stage_base, const __nv_bfloat16 *Kp, const __nv_bfloat16 *Vp,
-                                            const __nv_bfloat16 *kn, const __nv_bfloat16 *vn, int kb, int k1,
-                                            int Lapp, int g, int c, int lane)
-{
-    constexpr int NKI = D / 32, NVI = D / 64;
-#pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-        const int j = kb + 8 * nt + g;
-        const __nv_bfloat16 *row = (j == Lapp) ? kn : Kp + (long)(j < k1 ? j : 0) * D;
-        const int nbytes = j < k1 ? 16 : 0;
-#pragma unroll
-        for (int i = 0; i < NKI; ++i)
-            cp_async16(stage_base + ((nt * NKI + i) * 32 + lane) * 16, row + 8 * c + 32 * i, nbytes);
-    }
-#pragma unroll
-    for (int x = 0; x < 4; ++x) {
-        const int j = kb + 2 * c + (x & 1) + 8 * (x >> 1);
-        const __nv_bfloat16 *row = (j == Lapp) ? vn : Vp + (long)(j < k1 ? j : 0) * D;
-        const int nbytes = j < k1 ? 16 : 0;
-#pragma unroll
-        for (int i = 0; i < NVI; ++i)
-            cp_async16(stage_base + ((2 * NKI + x * NVI + i) * 32 + lane) * 16, row + 8 * g + 64 * i, nbytes);
-    }
-}
-
 __device__ __forceinline__ uint4 lds_u4(uint32_t addr)
 {
     uint4 r;
@@ -246,29 +208,91 @@ __device__ __forceinline__ uint4 lds_u4(uint32_t addr)
     return r;
 }
 
-constexpr int kDecodeStages = 3;
-constexpr int kDecodeWarps = 4;
+__device__ __forceinline__ void sts_u4(uint32_t addr, uint4 v)
+{
+    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// 2-D TMA tile load (x = element column, y = row) into shared memory, completing on bar.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+constexpr int kDecodeWarps = 8;       // warps per CTA (one CTA per SM)
+constexpr int kDecodeStages = 3;      // ring stages per warp
+constexpr int kMaxTmaUnits = 4096;    // plan entries kept in shared memory
+constexpr long long kSpinLimit = 1LL << 24;  // bounded mbarrier waits (about a second)
+
+template <int D> struct TmaLayout {
+    static constexpr int HALVES = D / 64;             // 128-byte boxes per row
+    static constexpr int TILE = 16 * 128;             // one 16-row box
+    static constexpr int STAGE = 4 * HALVES * 16 * 64; // K boxes then V boxes (bytes)
+    static constexpr int RING = kDecodeWarps * kDecodeStages * STAGE;
+};
 
 template <int D>
-__global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
+size_t tma_smem_bytes(int units)
 {
-    constexpr int NW = kDecodeWarps;
-    constexpr int NKI = D / 32;  // 16-byte K pieces per row per thread
-    constexpr int NVI = D / 64;  // 16-byte V pieces per row per thread
-    constexpr int KS = D / 16;   // k-steps of QK^T
-    constexpr int MT = D / 16;   // m-tiles of PV (d on M)
-    // dynamic shared memory: the per-warp cp.async rings, then the work plan
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    constexpr int RING_BYTES = kDecodeStages * (2 * NKI + 4 * NVI) * 32 * 16;
-    const uint32_t ring_base = (uint32_t)__cvta_generic_to_shared(smem_raw);
-    int *sm_pre = reinterpret_cast<int *>(smem_raw + NW * RING_BYTES);  // [units + 1] first item of each unit
-    int *sm_len = sm_pre + a.units + 1;  // [units] effective length (-1: invalid unit)
+    return 1024 + (size_t)TmaLayout<D>::RING + (size_t)(units + 1) * sizeof(int);
+}
+
+// Byte offset of 16-byte chunk ch (0..7) of row rr inside a 128B-swizzled 16-row box.
+__device__ __forceinline__ uint32_t swz(int rr, int ch) { return rr * 128 + ((ch ^ (rr & 7)) << 4); }
+
+template <int D>
+__global__ void __launch_bounds__(kDecodeWarps * 32, 1)
+    decode_tma(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, DecodeArgs a)
+{
+    using LY = TmaLayout<D>;
+    constexpr int NW = kDecodeWarps, S = kDecodeStages, HALVES = LY::HALVES, TILE = LY::TILE;
+    constexpr int STAGE = LY::STAGE;
+    constexpr int MT = D / 16;  // m-tiles of PV (d on M)
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t bars[NW][S];
     __shared__ long long sm_red[NW];
-    __shared__ int sm_scan[NW * 32 + 1];
+    __shared__ int sm_scan[NW];
+    const uint32_t raw0 = (uint32_t)__cvta_generic_to_shared(smem_raw);
+    const uint32_t ring0 = (raw0 + 1023u) & ~1023u;
+    int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
+    const uint32_t my_ring = ring0 + (uint32_t)wid * S * STAGE;
+    if (lane == 0) {
+        for (int s2 = 0; s2 < S; ++s2) mbar_init((uint32_t)__cvta_generic_to_shared(&bars[wid][s2]), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        fence_async_shared();
+    }
+    __syncwarp();
 
-    // ---- plan: identical in every CTA
+    // ---- plan: identical in every CTA (lens are not modified until every warp is done)
     const int seg = (units + blockDim.x - 1) / blockDim.x;
     const int u_lo = min(units, tid * seg), u_hi = min(units, u_lo + seg);
     long long tot = 0;
@@ -276,7 +300,6 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
         const int L = a.lens[u];
         const bool ok = unit_ok(L, a.L_cap, a.append);
         if (!ok && blockIdx.x == 0) raise_error(a.err, (a.append && L == a.L_cap) ? ERR_ROOM : ERR_LEN);
-        sm_len[u] = ok ? L + a.append : -1;
         tot += ok ? L + a.append : 0;
     }
 #pragma unroll
@@ -284,34 +307,32 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
     if (lane == 0) sm_red[wid] = tot;
     __syncthreads();
     tot = 0;
-    for (int w = 0; w < NW; ++w) tot += sm_red[w];
+    for (int w2 = 0; w2 < NW; ++w2) tot += sm_red[w2];
     const int total_warps = gridDim.x * NW;
-    const long long target = min((long long)kDecodeMaxTarget, 4LL * total_warps);
+    const long long target = min((long long)kDecodeMaxTarget, 8LL * total_warps);
     long long C = (tot + target - 1) / target;
     C = ((C + 63) / 64) * 64;
     if (C < 256) C = 256;
+    auto eff_len = [&](int u) {
+        const int L = a.lens[u];
+        return unit_ok(L, a.L_cap, a.append) ? L + a.append : -1;
+    };
     int my_items = 0;
-    for (int u = u_lo; u < u_hi; ++u) {
-        const int le = max(sm_len[u], 0);
-        my_items += max(1, (int)((le + C - 1) / C));
-    }
-    // exclusive scan of my_items over the block
+    for (int u = u_lo; u < u_hi; ++u) my_items += max(1, (int)((max(eff_len(u), 0) + C - 1) / C));
     {
         int incl = my_items;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            int n = __shfl_up_sync(0xffffffffu, incl, o);
+            const int n = __shfl_up_sync(0xffffffffu, incl, o);
             if (lane >= o) incl += n;
         }
         if (lane == 31) sm_scan[wid] = incl;
         __syncthreads();
-        int wbase = 0;
-        for (int w = 0; w < wid; ++w) wbase += sm_scan[w];
-        int run = wbase + incl - my_items;
+        int run = incl - my_items;
+        for (int w2 = 0; w2 < wid; ++w2) run += sm_scan[w2];
         for (int u = u_lo; u < u_hi; ++u) {
             sm_pre[u] = run;
-            const int le = max(sm_len[u], 0);
-            run += max(1, (int)((le + C - 1) / C));
+            run += max(1, (int)((max(eff_len(u), 0) + C - 1) / C));
         }
         if (tid == blockDim.x - 1) sm_pre[units] = run;
     }
@@ -319,6 +340,8 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
     const int total_items = sm_pre[units];
     const int g = lane >> 2, c = lane & 3;
     const bool out_bf16 = a.out_bf16 != 0;
+    uint32_t gblk = 0;  // 16-key blocks this warp has pushed through its ring
+    bool aborted = false;
 
     for (;;) {
         int item = 0;
@@ -333,7 +356,7 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
         const int u = lo;
         const int first = sm_pre[u], nsplit = sm_pre[u + 1] - first;
         const int split = item - first;
-        const int le_raw = sm_len[u];
+        const int le_raw = eff_len(u);
         const bool valid = le_raw >= 0;
         const int le = valid ? le_raw : 0;
         const int Lapp = (valid && a.append) ? le - 1 : -1;  // index of the appended row
@@ -342,62 +365,105 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
         const long lb = u / a.Hkv;
         const int h = u % a.Hkv;
         const int G = a.G;
-        const __nv_bfloat16 *Kp = reinterpret_cast<const __nv_bfloat16 *>(a.K) + (long)u * a.L_cap * D;
-        const __nv_bfloat16 *Vp = reinterpret_cast<const __nv_bfloat16 *>(a.V) + (long)u * a.L_cap * D;
-        const __nv_bfloat16 *kn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.k_new) + (long)u * D : Kp;
-        const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)u * D : Vp;
+        const __nv_bfloat16 *kn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.k_new) + (long)u * D : nullptr;
+        const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)u * D : nullptr;
         const long qrow0 = lb * a.Hq + (long)h * G;
+        const int row0 = u * a.L_cap;  // first tensor-map row of this unit
 
-        // Q fragments (rows g < G), head dim permuted: k-step j takes elements
-        // 8c + 32(j/2) + 4(j%2) + {0,1} (a0) and + {2,3} (a2).
-        uint32_t qa[KS][2];
+        // Q fragments (rows g < G), head dim permuted to match the K chunks: k-step
+        // j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
+        // and + {2,3} (a2).
+        uint32_t qa[D / 16][2];
         {
             const __nv_bfloat16 *qp = reinterpret_cast<const __nv_bfloat16 *>(a.q) + (qrow0 + g) * D;
 #pragma unroll
-            for (int i = 0; i < NKI; ++i) {
-                uint4 wv = make_uint4(0, 0, 0, 0);
-                if (g < G) wv = *reinterpret_cast<const uint4 *>(qp + 8 * c + 32 * i);
-                qa[2 * i][0] = wv.x;
-                qa[2 * i][1] = wv.y;
-                qa[2 * i + 1][0] = wv.z;
-                qa[2 * i + 1][1] = wv.w;
-            }
+            for (int hh = 0; hh < HALVES; ++hh)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    uint4 wv = make_uint4(0, 0, 0, 0);
+                    if (g < G) wv = *reinterpret_cast<const uint4 *>(qp + 64 * hh + 16 * c + 8 * e);
+                    const int j = 4 * hh + 2 * e;
+                    qa[j][0] = wv.x;
+                    qa[j][1] = wv.y;
+                    qa[j + 1][0] = wv.z;
+                    qa[j + 1][1] = wv.w;
+                }
         }
         float o[MT][4];
 #pragma unroll
         for (int t = 0; t < MT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
         float m = -INFINITY, l = 0.f;
 
-        constexpr int NP = 2 * NKI + 4 * NVI;  // pieces per thread per block
-        const uint32_t ring = ring_base + (uint32_t)wid * (kDecodeStages * NP * 32 * 16);
         const int nblk = (k1 - k0 + 15) / 16;
+        const uint32_t blk0 = gblk;
+        auto issue = [&](int bi) {  // lane 0 only
+            const uint32_t slot = (blk0 + bi) % S;
+            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
+            const uint32_t dst = my_ring + slot * STAGE;
+            const int y = row0 + k0 + 16 * bi;
+            fence_async_shared();
+            mbar_expect_tx(bar, STAGE);
 #pragma unroll
-        for (int p = 0; p < kDecodeStages - 1; ++p) {
-            if (p < nblk)
-                issue_block<D>(ring + p * NP * 512, Kp, Vp, kn, vn, k0 + 16 * p, k1, Lapp, g, c, lane);
-            cp_async_commit();
-        }
-        for (int bi = 0; bi < nblk; ++bi) {
-            {
-                const int nb = bi + kDecodeStages - 1;
-                if (nb < nblk)
-                    issue_block<D>(ring + (nb % kDecodeStages) * NP * 512, Kp, Vp, kn, vn, k0 + 16 * nb, k1, Lapp,
-                                   g, c, lane);
-                cp_async_commit();
+            for (int hh = 0; hh < HALVES; ++hh) {
+                tma_load_2d(dst + hh * TILE, &tmK, 64 * hh, y, bar);
+                tma_load_2d(dst + (HALVES + hh) * TILE, &tmV, 64 * hh, y, bar);
             }
-            cp_async_wait<kDecodeStages - 1>();
+        };
+        if (lane == 0)
+            for (int p = 0; p < S - 1 && p < nblk; ++p) issue(p);
+        for (int bi = 0; bi < nblk; ++bi) {
+            __syncwarp();
+            if (lane == 0 && bi + S - 1 < nblk) issue(bi + S - 1);
+            const uint32_t slot = (blk0 + bi) % S;
+            const uint32_t parity = ((blk0 + bi) / S) & 1u;
+            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
+            long long spins = 0;
+            while (!mbar_try_wait(bar, parity)) {
+                if (++spins > kSpinLimit) break;
+            }
+            if (spins > kSpinLimit) {  // a copy never landed: report, drain what is in flight, stop
+                if (lane == 0) raise_error(a.err, ERR_INTERNAL);
+                for (int p = bi + 1; p < nblk && p < bi + S; ++p) {
+                    const uint32_t sl = (blk0 + p) % S, par = ((blk0 + p) / S) & 1u;
+                    const uint32_t b2 = (uint32_t)__cvta_generic_to_shared(&bars[wid][sl]);
+                    for (long long t2 = 0; t2 < kSpinLimit && !mbar_try_wait(b2, par); ++t2) {
+                    }
+                }
+                aborted = true;
+                break;
+            }
             const int kb = k0 + 16 * bi;
-            const uint32_t st = ring + (bi % kDecodeStages) * NP * 512 + lane * 16;
+            const uint32_t Ks = my_ring + slot * STAGE, Vs = Ks + HALVES * TILE;
+            // patch the stage: zero V rows past the item (K rows there are masked), and
+            // put the appended row (not yet in the cache) in place
+            if (kb + 16 > k1 || (Lapp >= kb && Lapp < kb + 16)) {
+                const int zr = max(k1 - kb, 0);
+                for (int p = lane; p < (16 - zr) * HALVES * 8; p += 32) {
+                    const int rr = zr + p / (HALVES * 8), ch = p % (HALVES * 8);
+                    sts_u4(Vs + (ch >> 3) * TILE + swz(rr, ch & 7), make_uint4(0, 0, 0, 0));
+                }
+                if (Lapp >= kb && Lapp < kb + 16 && lane < 2 * HALVES * 8) {
+                    const int rr = Lapp - kb;
+                    const bool isv = lane >= HALVES * 8;
+                    const int ch = isv ? lane - HALVES * 8 : lane;
+                    const uint4 val = *reinterpret_cast<const uint4 *>((isv ? vn : kn) + ch * 8);
+                    sts_u4((isv ? Vs : Ks) + (ch >> 3) * TILE + swz(rr, ch & 7), val);
+                }
+                __syncwarp();
+            }
             float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int i = 0; i < NKI; ++i) {
-                const uint4 k0v = lds_u4(st + (0 * NKI + i) * 512);
-                const uint4 k1v = lds_u4(st + (1 * NKI + i) * 512);
-                mma_bf16(s0, qa[2 * i][0], 0u, qa[2 * i][1], 0u, k0v.x, k0v.y);
-                mma_bf16(s1, qa[2 * i][0], 0u, qa[2 * i][1], 0u, k1v.x, k1v.y);
-                mma_bf16(s0, qa[2 * i + 1][0], 0u, qa[2 * i + 1][1], 0u, k0v.z, k0v.w);
-                mma_bf16(s1, qa[2 * i + 1][0], 0u, qa[2 * i + 1][1], 0u, k1v.z, k1v.w);
-            }
+            for (int hh = 0; hh < HALVES; ++hh)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const uint4 ka = lds_u4(Ks + hh * TILE + swz(g, 2 * c + e));
+                    const uint4 kc = lds_u4(Ks + hh * TILE + swz(8 + g, 2 * c + e));
+                    const int j = 4 * hh + 2 * e;
+                    mma_bf16(s0, qa[j][0], 0u, qa[j][1], 0u, ka.x, ka.y);
+                    mma_bf16(s1, qa[j][0], 0u, qa[j][1], 0u, kc.x, kc.y);
+                    mma_bf16(s0, qa[j + 1][0], 0u, qa[j + 1][1], 0u, ka.z, ka.w);
+                    mma_bf16(s1, qa[j + 1][0], 0u, qa[j + 1][1], 0u, kc.z, kc.w);
+                }
             // scores of query g for keys kb+2c, kb+2c+1, kb+8+2c, kb+9+2c
             const int kA = kb + 2 * c, kB = kb + 8 + 2 * c;
             const float x0 = (kA < k1) ? s0[0] * a.c2 : -INFINITY;
@@ -429,35 +495,32 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
             split_bf16(p0, p1, ph0, pl0);
             split_bf16(p2, p3, ph1, pl1);
 #pragma unroll
-            for (int i = 0; i < NVI; ++i) {
-                const uint4 v0 = lds_u4(st + (2 * NKI + 0 * NVI + i) * 512);
-                const uint4 v1 = lds_u4(st + (2 * NKI + 1 * NVI + i) * 512);
-                const uint4 v2 = lds_u4(st + (2 * NKI + 2 * NVI + i) * 512);
-                const uint4 v3 = lds_u4(st + (2 * NKI + 3 * NVI + i) * 512);
+            for (int hh = 0; hh < HALVES; ++hh) {
+                const uint4 v0 = lds_u4(Vs + hh * TILE + swz(2 * c, g));
+                const uint4 v1 = lds_u4(Vs + hh * TILE + swz(2 * c + 1, g));
+                const uint4 v2 = lds_u4(Vs + hh * TILE + swz(2 * c + 8, g));
+                const uint4 v3 = lds_u4(Vs + hh * TILE + swz(2 * c + 9, g));
 #pragma unroll
                 for (int x = 0; x < 4; ++x) {
                     const uint32_t W0 = word(v0, x), W1 = word(v1, x), W2 = word(v2, x), W3 = word(v3, x);
                     const uint32_t A0 = __byte_perm(W0, W1, 0x5410), A1 = __byte_perm(W0, W1, 0x7632);
                     const uint32_t A2 = __byte_perm(W2, W3, 0x5410), A3 = __byte_perm(W2, W3, 0x7632);
-                    mma_bf16(o[4 * i + x], A0, A1, A2, A3, ph0, ph1);
-                    mma_bf16(o[4 * i + x], A0, A1, A2, A3, pl0, pl1);
+                    mma_bf16(o[4 * hh + x], A0, A1, A2, A3, ph0, ph1);
+                    mma_bf16(o[4 * hh + x], A0, A1, A2, A3, pl0, pl1);
                 }
             }
         }
+        gblk += nblk;
+        if (aborted) break;
         l += __shfl_xor_sync(0xffffffffu, l, 1);
         l += __shfl_xor_sync(0xffffffffu, l, 2);
 
         // the warp that covers the appended index writes the new row into the cache
-        if (Lapp >= k0 && Lapp < k1) {
-            constexpr int PCS = D / 8;  // 16-byte pieces per row
-            if (lane < 2 * PCS) {
-                const bool isv = lane >= PCS;
-                const int pc = isv ? lane - PCS : lane;
-                const __nv_bfloat16 *src = (isv ? vn : kn) + pc * 8;
-                __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(isv ? a.V : a.K) +
-                                     ((long)u * a.L_cap + Lapp) * D + pc * 8;
-                *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
-            }
+        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8)) {
+            const bool isv = lane >= D / 8;
+            const int pc = isv ? lane - D / 8 : lane;
+            __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(isv ? a.V : a.K) + ((long)row0 + Lapp) * D + pc * 8;
+            *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>((isv ? vn : kn) + pc * 8);
         }
 
         const int q0 = 2 * c, q1 = 2 * c + 1;
@@ -465,17 +528,17 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
         if (nsplit == 1) {
             const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
 #pragma unroll
-            for (int i = 0; i < NVI; ++i) {
-                const long d0 = 64 * i + 8 * g;
+            for (int hh = 0; hh < HALVES; ++hh) {
+                const long d0 = 64 * hh + 8 * g;
 #pragma unroll
                 for (int x = 0; x < 4; ++x) {
                     if (q0 < G) {
-                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q0) * D + d0 + 2 * x, o[4 * i + x][0] * inv0);
-                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q0) * D + d0 + 2 * x + 1, o[4 * i + x][2] * inv0);
+                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q0) * D + d0 + 2 * x, o[4 * hh + x][0] * inv0);
+                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q0) * D + d0 + 2 * x + 1, o[4 * hh + x][2] * inv0);
                     }
                     if (q1 < G) {
-                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q1) * D + d0 + 2 * x, o[4 * i + x][1] * inv1);
-                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q1) * D + d0 + 2 * x + 1, o[4 * i + x][3] * inv1);
+                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q1) * D + d0 + 2 * x, o[4 * hh + x][1] * inv1);
+                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + q1) * D + d0 + 2 * x + 1, o[4 * hh + x][3] * inv1);
                     }
                 }
             }
@@ -483,17 +546,17 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
         } else {
             float *po = a.part_o + (size_t)item * G * D;
 #pragma unroll
-            for (int i = 0; i < NVI; ++i) {
-                const int d0 = 64 * i + 8 * g;
+            for (int hh = 0; hh < HALVES; ++hh) {
+                const int d0 = 64 * hh + 8 * g;
                 if (q0 < G) {
                     float4 *dst = reinterpret_cast<float4 *>(po + (size_t)q0 * D + d0);
-                    dst[0] = make_float4(o[4 * i + 0][0], o[4 * i + 0][2], o[4 * i + 1][0], o[4 * i + 1][2]);
-                    dst[1] = make_float4(o[4 * i + 2][0], o[4 * i + 2][2], o[4 * i + 3][0], o[4 * i + 3][2]);
+                    dst[0] = make_float4(o[4 * hh + 0][0], o[4 * hh + 0][2], o[4 * hh + 1][0], o[4 * hh + 1][2]);
+                    dst[1] = make_float4(o[4 * hh + 2][0], o[4 * hh + 2][2], o[4 * hh + 3][0], o[4 * hh + 3][2]);
                 }
                 if (q1 < G) {
                     float4 *dst = reinterpret_cast<float4 *>(po + (size_t)q1 * D + d0);
-                    dst[0] = make_float4(o[4 * i + 0][1], o[4 * i + 0][3], o[4 * i + 1][1], o[4 * i + 1][3]);
-                    dst[1] = make_float4(o[4 * i + 2][1], o[4 * i + 2][3], o[4 * i + 3][1], o[4 * i + 3][3]);
+                    dst[0] = make_float4(o[4 * hh + 0][1], o[4 * hh + 0][3], o[4 * hh + 1][1], o[4 * hh + 1][3]);
+                    dst[1] = make_float4(o[4 * hh + 2][1], o[4 * hh + 2][3], o[4 * hh + 3][1], o[4 * hh + 3][3]);
                 }
             }
             if (c == 0 && g < G) {
@@ -510,16 +573,15 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
                 constexpr int PER = D / 32;
                 for (int qq = 0; qq < G; ++qq) {
                     float M = -INFINITY;
-                    for (int s = 0; s < nsplit; ++s)
-                        M = fmaxf(M, __ldcg(a.part_ml + ((size_t)(first + s) * G + qq) * 2));
+                    for (int s2 = 0; s2 < nsplit; ++s2)
+                        M = fmaxf(M, __ldcg(a.part_ml + ((size_t)(first + s2) * G + qq) * 2));
                     float Ls = 0.f, acc[PER];
 #pragma unroll
                     for (int e = 0; e < PER; ++e) acc[e] = 0.f;
                     if (M != -INFINITY) {
-                        for (int s = 0; s < nsplit; ++s) {
-                            const size_t it = (size_t)(first + s) * G + qq;
-                            const float ms = __ldcg(a.part_ml + it * 2);
-                            const float wt = fast_exp2(ms - M);
+                        for (int s2 = 0; s2 < nsplit; ++s2) {
+                            const size_t it = (size_t)(first + s2) * G + qq;
+                            const float wt = fast_exp2(__ldcg(a.part_ml + it * 2) - M);
                             Ls += __ldcg(a.part_ml + it * 2 + 1) * wt;
                             const float *src = a.part_o + it * D + lane * PER;
 #pragma unroll
@@ -535,24 +597,51 @@ __global__ void __launch_bounds__(128, 2) decode_mma(DecodeArgs a)
             }
         }
     }
+    if (aborted) return;
     // the last warp of the grid advances the lengths (every plan has been read by then)
     int done = 0;
     if (lane == 0) done = atomicAdd(&a.counters[1], 1);
     done = __shfl_sync(0xffffffffu, done, 0);
     if (done == total_warps - 1 && a.append) {
         __threadfence();
-        for (int u = lane; u < units; u += 32)
-            if (sm_len[u] >= 0) a.lens[u] = sm_len[u];
+        for (int u = lane; u < units; u += 32) {
+            const int le = eff_len(u);
+            if (le >= 0) a.lens[u] = le;
+        }
     }
 }
 
-constexpr int kMaxMmaUnits = 8192;  // plan (8 B per unit) + rings stay within one CTA's shared memory
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-static int mma_blocks_per_sm(const void *fn, size_t smem)
+static EncodeTiledFn encode_fn()
 {
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, 128, smem) != cudaSuccess || n < 1) n = 1;
-    return n;
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)p;
+    }
+    return fn;
+}
+
+// [rows, d] bf16 view of a cache tensor, 16-row x 64-column boxes, 128-byte swizzle.
+static bool encode_cache_map(CUtensorMap *map, const void *base, unsigned long long rows, int d)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+    const cuuint32_t box[2] = {64, 16};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
@@ -581,20 +670,23 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.out_bf16 = out_dtype == RECO_BF16 ? 1 : 0;
     a.c2 = scale * kLog2e;
     a.err = err;
-    if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxMmaUnits) {
-        cudaError_t e = cudaMemsetAsync(ws.counters, 0, (size_t)(2 + a.units) * 4, s);
-        if (e != cudaSuccess) return e;
-        const size_t ring = (size_t)kDecodeWarps * kDecodeStages * (kv.d == 64 ? 8 : 16) * 32 * 16;
-        const size_t smem = ring + (size_t)(2 * a.units + 1) * sizeof(int);
-        const void *fn = kv.d == 64 ? (const void *)decode_mma<64> : (const void *)decode_mma<128>;
-        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        const int grid = device_sm_count() * mma_blocks_per_sm(fn, smem);
-        if (kv.d == 64)
-            decode_mma<64><<<grid, 128, smem, s>>>(a);
-        else
-            decode_mma<128><<<grid, 128, smem, s>>>(a);
-        return cudaGetLastError();
+    const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
+    if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31)) {
+        CUtensorMap mk, mv;
+        if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {
+            cudaError_t e = cudaMemsetAsync(ws.counters, 0, (size_t)(2 + a.units) * 4, s);
+            if (e != cudaSuccess) return e;
+            const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(a.units) : tma_smem_bytes<128>(a.units);
+            const void *fn = kv.d == 64 ? (const void *)decode_tma<64> : (const void *)decode_tma<128>;
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+            const int grid = device_sm_count();
+            if (kv.d == 64)
+                decode_tma<64><<<grid, kDecodeWarps * 32, smem, s>>>(mk, mv, a);
+            else
+                decode_tma<128><<<grid, kDecodeWarps * 32, smem, s>>>(mk, mv, a);
+            return cudaGetLastError();
+        }
     }
     const unsigned grid = (unsigned)a.units;
     if (kv.dtype == RECO_F32) {

@@ -11,7 +11,7 @@ namespace reco {
 // Keys per scoring work item (one CTA per (unit, chunk) in both scoring passes).
 constexpr int kScoreChunk = 2048;
 // Upper bound on decode split-K work items beyond one per unit.
-constexpr int kDecodeMaxTarget = 8192;
+constexpr int kDecodeMaxTarget = 16384;
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
