@@ -59,4 +59,10 @@ cudaError_t launch_ppl(const float *logits, const int32_t *tokens, const int32_t
 // Device properties cached per device.
 int device_sm_count();
 
+// Encode a 2-D tensor map over a row-major bf16 matrix [rows, cols] with boxes of
+// box_rows x box_cols elements and 128-byte swizzle (box_cols * 2 <= 128).
+// Returns false if the driver entry point is unavailable or the encode fails.
+bool encode_bf16_2d(void *map /* CUtensorMap */, const void *base, unsigned long long rows, int cols,
+                    int box_cols, int box_rows);
+
 }  // namespace reco

@@ -9,8 +9,9 @@
 //   combine per (unit, row): merge the chunk partials -> b_r = m_r + log2 Z_r
 //   pass 2  per (unit, key chunk): column sums  sum_r 2^(c*l_rj - b_r) / G
 //   pool    per (unit, key): max over the clipped window
-// This file holds the SIMT version used for float32 caches (and any shape the
-// tensor-core version does not cover); score_tc.cu holds the bf16 tensor-core passes.
+// This file holds the SIMT passes used for float32 caches (and any shape the tensor-
+// core passes do not cover), the combine and pool kernels, and the launcher;
+// score_tc.cu holds the bf16 tensor-core (tcgen05) passes.
 #include "common.cuh"
 #include "internal.h"
 
@@ -197,8 +198,11 @@ __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restr
     scores[u * L_cap + j] = m;
 }
 
-cudaError_t launch_score_tc(const reco_kv &kv, const void *q_win, const int32_t *lens, int w,
-                            float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+bool score_tc_supported(const reco_kv &kv, int w);
 
 template <typename T, int D>
 static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *lens, int w, float c2,
@@ -233,6 +237,7 @@ constexpr size_t kSimtMaxQ = 200 * 1024 / 4;
 bool score_shape_supported(const reco_kv &kv, int w)
 {
     size_t R = (size_t)(kv.H_q / kv.H_kv) * w;
+    if (score_tc_supported(kv, w)) return true;
     return (kv.d == 64 || kv.d == 128) && (R * kv.d + R) <= kSimtMaxQ;
 }
 
@@ -243,8 +248,21 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
     cudaError_t e = cudaSuccess;
     bool used_tc = false;
     if (kv.dtype == RECO_BF16) {
-        e = launch_score_tc(kv, q_win, lens, w, c2, ws, err, s, &used_tc);
+        // tensor-core passes: pass 1 -> combine -> pass 2
+        e = launch_score_tc_pass1(kv, q_win, lens, w, c2, ws, err, s, &used_tc);
         if (e != cudaSuccess) return e;
+        if (used_tc) {
+            const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+            const int R = (kv.H_q / kv.H_kv) * w;
+            const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
+            score_combine<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, w, kv.L_cap, R, nch, ws.part_m,
+                                                                              ws.part_z, ws.rowb, units);
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+            bool used2 = false;
+            e = launch_score_tc_pass2(kv, q_win, lens, w, c2, ws, err, s, &used2);
+            if (e != cudaSuccess) return e;
+            if (!used2) return cudaErrorNotSupported;
+        }
     }
     if (!used_tc) {
         if (kv.dtype == RECO_F32)

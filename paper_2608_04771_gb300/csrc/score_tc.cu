@@ -1,15 +1,504 @@
 // score_tc.cu -- tensor-core (tcgen05) passes of the Eq. 2 cache scores for bf16 caches.
+//
+// Both passes run one CTA per (unit, 2048-key chunk) with the same roles:
+//   warp 0  lane 0 : TMA producer (window queries once, then a ring of K tiles)
+//   warp 1         : allocates 512 TMEM columns; lane 0 issues tcgen05.mma (bf16 in,
+//                    fp32 accumulate in TMEM) and commits to mbarriers
+//   warps 4.. 	    : epilogue, reading accumulators with tcgen05.ld (one TMEM lane
+//                    per thread) into the softmax arithmetic
+// Operands sit in shared memory in the 128-byte-swizzled K-major layout the TMA writes
+// (rows of 64 bf16, 8-row atoms of 1024 bytes); each MMA takes a K=16 slice.
+//
+// Pass 1 (row statistics): queries on M (128-row tiles), keys on N, so each thread
+//   owns one window row and keeps its running max / sum over the chunk's keys.
+// Pass 2 (column sums): keys on M (128 per tile), queries on N, so each thread owns
+//   one key and sums 2^(c*l - b_r) over the window rows with b_r from pass 1.
+// Every mbarrier wait is bounded; a wait that runs out sets the device error word and
+// the CTA stops issuing work, waits (bounded) for nothing further and frees its TMEM.
+#include <cuda.h>
+
 #include "common.cuh"
 #include "internal.h"
+#include "tma.cuh"
 
 namespace reco {
 
-cudaError_t launch_score_tc(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                            const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+// ---------------------------------------------------------------- tcgen05 wrappers
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols)
 {
-    (void)kv; (void)q_win; (void)lens; (void)w; (void)c2; (void)ws; (void)err; (void)s;
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish()
+{
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
+{
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, kind::f16 (both operands bf16 here).
+__device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate)
+{
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(dtmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// 32 consecutive fp32 columns of the calling thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row atoms of
+// 1024 bytes (stride byte offset 1024), descriptor version 1.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)1u << 16;            // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024u >> 4) << 32;  // stride byte offset
+    d |= (uint64_t)1u << 46;            // version
+    d |= (uint64_t)2u << 61;            // SWIZZLE_128B
+    return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
+{
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+constexpr long long kTcSpin = 1LL << 24;
+constexpr int kTmemCols = 512;
+
+__device__ __forceinline__ bool wait_or_flag(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                             unsigned *err)
+{
+    for (long long i = 0; i < kTcSpin; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 1023) == 1023 && *abort_flag) return false;
+    }
+    *abort_flag = 1;
+    raise_error(err, ERR_INTERNAL);
+    return false;
+}
+
+// ---------------------------------------------------------------- pass 1: row statistics
+template <int D, int N, int MT>
+__global__ void __launch_bounds__(128 + 128 * MT, 1)
+    score_rowstats_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                      const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R,
+                      int n_chunks, float c2, float *__restrict__ part_m, float *__restrict__ part_z,
+                      unsigned *err)
+{
+    constexpr int HALVES = D / 64;
+    constexpr int QBOX = 128 * 128;  // 128 rows x 128 bytes
+    constexpr int KBOX = N * 128;
+    constexpr int KSTAGE = HALVES * KBOX;
+    constexpr int NS = 4;
+    constexpr uint32_t IDESC = idesc_bf16(128, N);
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t bar_q, bar_kfull[NS], bar_kempty[NS], bar_afull[2], bar_aempty[2];
+    __shared__ uint32_t tmem_sh;
+    __shared__ int abort_sh;
+
+    const int chunk = blockIdx.x;
+    const long u = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int L = lens[u];
+    if (L < w || L > L_cap) {
+        if (chunk == 0 && tid == 0) raise_error(err, ERR_LEN);
+        return;
+    }
+    const int j0 = chunk * kScoreChunk;
+    const int j1 = min(j0 + kScoreChunk, L);
+    const int ntiles = j0 < j1 ? (j1 - j0 + N - 1) / N : 0;
+    if (ntiles == 0) {  // chunk past the end: empty statistics
+        for (int r = tid; r < R; r += blockDim.x) {
+            part_m[((size_t)u * n_chunks + chunk) * R + r] = -INFINITY;
+            part_z[((size_t)u * n_chunks + chunk) * R + r] = 0.f;
+        }
+        return;
+    }
+    const uint32_t raw0 = smem_addr(smem_raw);
+    const uint32_t base = (raw0 + 1023u) & ~1023u;
+    const uint32_t Qs = base;                                  // MT x HALVES x QBOX
+    const uint32_t Ks = base + (uint32_t)MT * HALVES * QBOX;  // NS x KSTAGE
+    if (tid == 0) {
+        mbar_init(smem_addr(&bar_q), 1);
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(smem_addr(&bar_kfull[s]), 1);
+            mbar_init(smem_addr(&bar_kempty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_addr(&bar_afull[b]), 1);
+            mbar_init(smem_addr(&bar_aempty[b]), 4 * MT);
+        }
+        abort_sh = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        fence_async_shared();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&tmem_sh), kTmemCols);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+    const long lb = u / Hkv;
+    const int h = (int)(u % Hkv);
+    const int q_row0 = (int)((lb * Hq + (long)h * G) * w);
+    const int k_row0 = (int)(u * L_cap + j0);
+    volatile int *abort_flag = &abort_sh;
+
+    if (warp == 0) {
+        if (lane == 0) {  // producer
+            mbar_expect_tx(smem_addr(&bar_q), (uint32_t)MT * HALVES * QBOX);
+            for (int mt = 0; mt < MT; ++mt)
+                for (int hh = 0; hh < HALVES; ++hh)
+                    tma_load_2d(Qs + (mt * HALVES + hh) * QBOX, &tmQ, 64 * hh, q_row0 + 128 * mt, smem_addr(&bar_q));
+            for (int t = 0; t < ntiles; ++t) {
+                const int s = t % NS;
+                const uint32_t ph = (t / NS) & 1;
+                if (!wait_or_flag(smem_addr(&bar_kempty[s]), ph ^ 1, abort_flag, err)) break;
+                mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
+                for (int hh = 0; hh < HALVES; ++hh)
+                    tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * N, smem_addr(&bar_kfull[s]));
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // MMA issuer
+            bool ok = wait_or_flag(smem_addr(&bar_q), 0, abort_flag, err);
+            for (int t = 0; ok && t < ntiles; ++t) {
+                const int s = t % NS, b = t & 1;
+                const uint32_t ph = (t / NS) & 1, bph = (t >> 1) & 1;
+                if (!wait_or_flag(smem_addr(&bar_kfull[s]), ph, abort_flag, err)) break;
+                if (!wait_or_flag(smem_addr(&bar_aempty[b]), bph ^ 1, abort_flag, err)) break;
+                tc_fence_after();
+                for (int mt = 0; mt < MT; ++mt) {
+                    const uint32_t d = tmem + (uint32_t)((b * MT + mt) * N);
+#pragma unroll
+                    for (int k = 0; k < D / 16; ++k) {
+                        const int hh = k >> 2, kk = k & 3;
+                        const uint64_t ad = sw128_desc(Qs + (mt * HALVES + hh) * QBOX + kk * 32);
+                        const uint64_t bd = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
+                        tc_mma(d, ad, bd, IDESC, k > 0 ? 1u : 0u);
+                    }
+                }
+                tc_commit(smem_addr(&bar_kempty[s]));
+                tc_commit(smem_addr(&bar_afull[b]));
+            }
+        }
+    } else if (warp >= 4 && warp < 4 + 4 * MT) {  // epilogue: one window row per thread
+        const int e = warp - 4, mt = e >> 2, quarter = warp & 3;
+        const int r = mt * 128 + quarter * 32 + lane;
+        const int t_row = r % w;
+        const int jmax = L - w + t_row;  // last key this window row sees
+        float m = -INFINITY, z = 0.f;
+        for (int t = 0; t < ntiles; ++t) {
+            const int b = t & 1;
+            const uint32_t bph = (t >> 1) & 1;
+            if (!wait_or_flag(smem_addr(&bar_afull[b]), bph, abort_flag, err)) break;
+            tc_fence_after();
+            const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((b * MT + mt) * N);
+            const int jb = j0 + t * N;
+            const int lim = min(j1 - 1, jmax) - jb;  // columns 0..lim are visible to this row
+#pragma unroll 1
+            for (int cc = 0; cc < N; cc += 32) {
+                float v[32];
+                tmem_ld32(ta + cc, v);
+                float mx = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    v[i] *= c2;
+                    if (cc + i <= lim) mx = fmaxf(mx, v[i]);
+                }
+                const float mn = fmaxf(m, mx);
+                if (mn == -INFINITY) continue;
+                float acc = 0.f;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) acc += (cc + i <= lim) ? fast_exp2(v[i] - mn) : 0.f;
+                z = z * fast_exp2(m - mn) + acc;
+                m = mn;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
+        }
+        if (r < R && !*abort_flag) {
+            part_m[((size_t)u * n_chunks + chunk) * R + r] = m;
+            part_z[((size_t)u * n_chunks + chunk) * R + r] = z;
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------- pass 2: column sums
+// NQ (runtime, multiple of 16, <= 512) query columns per tile.  With NQ <= 256 the two
+// epilogue warpgroups take alternate tiles (two TMEM buffers); above 256 one buffer is
+// shared and each warpgroup sums half of the columns.
+template <int D>
+__global__ void __launch_bounds__(128 + 256, 1)
+    score_colsum_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R, int NQ,
+                    float c2, const float *__restrict__ rowb, float *__restrict__ raw, unsigned *err)
+{
+    constexpr int HALVES = D / 64;
+    constexpr int KBOX = 128 * 128;  // 128 keys x 128 bytes
+    constexpr int KSTAGE = HALVES * KBOX;
+    constexpr int NS = 3;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t bar_q, bar_kfull[NS], bar_kempty[NS], bar_afull[2], bar_aempty[2];
+    __shared__ uint32_t tmem_sh;
+    __shared__ int abort_sh;
+    __shared__ float bsh[512];
+
+    const int chunk = blockIdx.x;
+    const long u = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int L = lens[u];
+    if (L < w || L > L_cap) return;
+    const int nc = L - w;
+    const int j0 = chunk * kScoreChunk;
+    const int j1 = min(j0 + kScoreChunk, nc);
+    if (j0 >= j1) return;
+    const int ntiles = (j1 - j0 + 127) / 128;
+    const bool split_cols = NQ > 256;
+    const int NBUF = split_cols ? 1 : 2;
+    const int nmma = split_cols ? 2 : 1;
+    const int NM = NQ / nmma;  // MMA N
+    const uint32_t idesc = idesc_bf16(128, NM);
+    const uint32_t raw0 = smem_addr(smem_raw);
+    const uint32_t base = (raw0 + 1023u) & ~1023u;
+    const uint32_t QBOXB = (uint32_t)NQ * 128;  // one half (64 columns) of all NQ query rows
+    const uint32_t Qs = base;
+    const uint32_t Ks = base + HALVES * QBOXB;
+    for (int r = tid; r < 512; r += blockDim.x) bsh[r] = r < R ? rowb[u * R + r] : 0.f;
+    if (tid == 0) {
+        mbar_init(smem_addr(&bar_q), 1);
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(smem_addr(&bar_kfull[s]), 1);
+            mbar_init(smem_addr(&bar_kempty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_addr(&bar_afull[b]), 1);
+            mbar_init(smem_addr(&bar_aempty[b]), split_cols ? 8 : 4);
+        }
+        abort_sh = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        fence_async_shared();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&tmem_sh), kTmemCols);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+    const long lb = u / Hkv;
+    const int h = (int)(u % Hkv);
+    const int q_row0 = (int)((lb * Hq + (long)h * G) * w);
+    const int k_row0 = (int)(u * L_cap + j0);
+    volatile int *abort_flag = &abort_sh;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const int qbox_rows = NQ > 256 ? NQ / 2 : NQ;
+            mbar_expect_tx(smem_addr(&bar_q), HALVES * QBOXB);
+            for (int hh = 0; hh < HALVES; ++hh)
+                for (int r0 = 0; r0 < NQ; r0 += qbox_rows)
+                    tma_load_2d(Qs + hh * QBOXB + r0 * 128, &tmQ, 64 * hh, q_row0 + r0, smem_addr(&bar_q));
+            for (int t = 0; t < ntiles; ++t) {
+                const int s = t % NS;
+                const uint32_t ph = (t / NS) & 1;
+                if (!wait_or_flag(smem_addr(&bar_kempty[s]), ph ^ 1, abort_flag, err)) break;
+                mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
+                for (int hh = 0; hh < HALVES; ++hh)
+                    tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * 128, smem_addr(&bar_kfull[s]));
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            bool ok = wait_or_flag(smem_addr(&bar_q), 0, abort_flag, err);
+            for (int t = 0; ok && t < ntiles; ++t) {
+                const int s = t % NS, b = NBUF == 2 ? (t & 1) : 0;
+                const uint32_t ph = (t / NS) & 1, bph = NBUF == 2 ? ((t >> 1) & 1) : (t & 1);
+                if (!wait_or_flag(smem_addr(&bar_kfull[s]), ph, abort_flag, err)) break;
+                if (!wait_or_flag(smem_addr(&bar_aempty[b]), bph ^ 1, abort_flag, err)) break;
+                tc_fence_after();
+                for (int nb = 0; nb < nmma; ++nb) {
+                    const uint32_t d = tmem + (uint32_t)(b * 256 + nb * NM);
+                    for (int k = 0; k < D / 16; ++k) {
+                        const int hh = k >> 2, kk = k & 3;
+                        const uint64_t ad = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
+                        const uint64_t bd = sw128_desc(Qs + hh * QBOXB + nb * NM * 128 + kk * 32);
+                        tc_mma(d, ad, bd, idesc, k > 0 ? 1u : 0u);
+                    }
+                }
+                tc_commit(smem_addr(&bar_kempty[s]));
+                tc_commit(smem_addr(&bar_afull[b]));
+            }
+        }
+    } else if (warp >= 4) {  // epilogue: one key per thread
+        const int eg = (warp - 4) >> 2, quarter = warp & 3;
+        const int row = quarter * 32 + lane;  // key within the tile
+        const int c_lo = split_cols ? eg * (NQ / 2) : 0;
+        const int c_hi = split_cols ? c_lo + NQ / 2 : NQ;
+        const float invG = 1.f / (float)G;
+        for (int t = split_cols ? 0 : eg; t < ntiles; t += split_cols ? 1 : 2) {
+            const int b = NBUF == 2 ? (t & 1) : 0;
+            const uint32_t bph = NBUF == 2 ? ((t >> 1) & 1) : (t & 1);
+            if (!wait_or_flag(smem_addr(&bar_afull[b]), bph, abort_flag, err)) break;
+            tc_fence_after();
+            const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * 256);
+            float acc = 0.f;
+            for (int cb = c_lo; cb < c_hi; cb += 32) {
+                float v[32];
+                tmem_ld32(ta + cb, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (cb + i < R) acc += fast_exp2(fmaf(v[i], c2, -bsh[cb + i]));
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
+            const int j = j0 + t * 128 + row;
+            if (j < j1) {
+                if (split_cols)  // two halves land on a zeroed entry: 0 + a + b, order-independent
+                    atomicAdd(raw + u * L_cap + j, acc * invG);
+                else
+                    raw[u * L_cap + j] = acc * invG;
+            }
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------- host side
+constexpr int kTcMaxR = 448;  // keeps pass 2 (queries + 3 K stages) within 227 KB of shared memory
+
+int score_tc_nq(int R) { return R <= 256 ? ((R + 15) / 16) * 16 : ((R + 31) / 32) * 32; }
+
+bool score_tc_supported(const reco_kv &kv, int w)
+{
+    const long long R = (long long)(kv.H_q / kv.H_kv) * w;
+    const unsigned long long k_rows = (unsigned long long)kv.n_layers * kv.B * kv.H_kv * kv.L_cap;
+    const unsigned long long q_rows = (unsigned long long)kv.n_layers * kv.B * kv.H_q * w;
+    return kv.dtype == RECO_BF16 && (kv.d == 64 || kv.d == 128) && R <= kTcMaxR && k_rows < (1ull << 31) &&
+           q_rows < (1ull << 31);
+}
+
+template <int D, int N, int MT>
+static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                             const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const int R = (kv.H_q / kv.H_kv) * w;
+    const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
+    const unsigned long long k_rows = (unsigned long long)units * kv.L_cap;
+    const unsigned long long q_rows = (unsigned long long)kv.n_layers * kv.B * kv.H_q * w;
+    CUtensorMap mq, mk;
+    if (!encode_bf16_2d(&mq, q_win, q_rows, D, 64, 128) || !encode_bf16_2d(&mk, kv.k, k_rows, D, 64, N)) {
+        *ok = false;
+        return cudaSuccess;
+    }
+    const size_t smem = 1024 + (size_t)MT * (D / 64) * 128 * 128 + 4 * (size_t)(D / 64) * N * 128;
+    cudaError_t e = cudaFuncSetAttribute(score_rowstats_tc<D, N, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    score_rowstats_tc<D, N, MT><<<dim3(nch, (unsigned)units), 128 + 128 * MT, smem, s>>>(
+        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, nch, c2, ws.part_m, ws.part_z, err);
+    *ok = true;
+    return cudaGetLastError();
+}
+
+template <int D>
+static cudaError_t pass1_by_mt(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                               const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+{
+    const int MT = ((kv.H_q / kv.H_kv) * w + 127) / 128;
+    switch (MT) {
+    case 1: return run_pass1<D, 128, 1>(kv, q_win, lens, w, c2, ws, err, s, ok);
+    case 2: return run_pass1<D, 128, 2>(kv, q_win, lens, w, c2, ws, err, s, ok);
+    case 3: return run_pass1<D, 64, 3>(kv, q_win, lens, w, c2, ws, err, s, ok);
+    default: return run_pass1<D, 64, 4>(kv, q_win, lens, w, c2, ws, err, s, ok);
+    }
+}
+
+cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+{
     *used = false;
-    return cudaSuccess;
+    if (!score_tc_supported(kv, w)) return cudaSuccess;
+    return kv.d == 128 ? pass1_by_mt<128>(kv, q_win, lens, w, c2, ws, err, s, used)
+                       : pass1_by_mt<64>(kv, q_win, lens, w, c2, ws, err, s, used);
+}
+
+template <int D>
+static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                             const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const int R = (kv.H_q / kv.H_kv) * w;
+    const int NQ = score_tc_nq(R);
+    const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
+    const unsigned long long k_rows = (unsigned long long)units * kv.L_cap;
+    const unsigned long long q_rows = (unsigned long long)kv.n_layers * kv.B * kv.H_q * w;
+    CUtensorMap mq, mk;
+    const int qbox = NQ > 256 ? NQ / 2 : NQ;
+    if (!encode_bf16_2d(&mq, q_win, q_rows, D, 64, qbox) || !encode_bf16_2d(&mk, kv.k, k_rows, D, 64, 128)) {
+        *ok = false;
+        return cudaSuccess;
+    }
+    cudaError_t e;
+    if (NQ > 256 && (e = cudaMemsetAsync(ws.raw, 0, (size_t)units * kv.L_cap * sizeof(float), s)) != cudaSuccess)
+        return e;
+    const size_t smem = 1024 + (size_t)(D / 64) * NQ * 128 + 3 * (size_t)(D / 64) * 128 * 128;
+    e = cudaFuncSetAttribute(score_colsum_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    score_colsum_tc<D><<<dim3(nch, (unsigned)units), 128 + 256, smem, s>>>(
+        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, NQ, c2, ws.rowb, ws.raw, err);
+    *ok = true;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
+                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+{
+    *used = false;
+    if (!score_tc_supported(kv, w)) return cudaSuccess;
+    return kv.d == 128 ? run_pass2<128>(kv, q_win, lens, w, c2, ws, err, s, used)
+                       : run_pass2<64>(kv, q_win, lens, w, c2, ws, err, s, used);
 }
 
 }  // namespace reco
