@@ -177,6 +177,23 @@ reco_status reco_answer_ppl(const float *logits, const int32_t *tokens, const in
                             int n, int V, float tau_p, float *ppl, uint8_t *stop, void *ws,
                             size_t ws_bytes, cudaStream_t stream);
 
+/* Allocation-free variant of reco_answer_ppl (the paper has no counterpart: this is
+ * a library convenience).  Same arguments and results as reco_answer_ppl, but the
+ * per-row scratch is a fixed array inside the library instead of a caller workspace,
+ * for callers that cannot allocate device memory (for example a plug-in whose host
+ * engine has reserved the whole GPU, or C code with no device allocator).
+ *   - B*n must not exceed RECO_PPL_STATIC_MAX_ROWS, else RECO_EINVAL (nothing runs).
+ *   - Allocates nothing: no cudaMalloc / cudaFree, no allocating library routine.
+ *   - The first call on each device looks up the array's device address (once, with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls on a device share the one array and it keeps the last call's
+ *     contents; every entry a call reads is written by that call first, so nothing
+ *     needs clearing, but calls whose executions overlap on the GPU race on it.
+ *   - Every GPU that loads the library holds the array (256 KB) until process exit. */
+#define RECO_PPL_STATIC_MAX_ROWS 65536
+reco_status reco_answer_ppl_static(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B,
+                                   int n, int V, float tau_p, float *ppl, uint8_t *stop, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

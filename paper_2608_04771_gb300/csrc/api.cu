@@ -317,3 +317,55 @@ reco_status reco_answer_ppl(const float *logits, const int32_t *tokens, const in
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- allocation-free answer PPL
+// Some callers cannot hand the library any device memory of their own: a plug-in
+// running inside a host engine that has already reserved every byte of the GPU for
+// its own pool, or plain C code that has no device allocator to call.  For them the
+// answer-PPL step can run on a fixed scratch array that lives in the library itself
+// (one float per answer row), so the caller passes only its inputs and outputs.
+// The array is part of the loaded module: every GPU that loads the library holds its
+// 256 KB until the process exits.
+static __device__ __align__(256) float g_ppl_static_rows[RECO_PPL_STATIC_MAX_ROWS];
+
+namespace {
+float *g_ppl_static_addr[128];
+
+// Device address of g_ppl_static_rows on the current device, looked up once per device
+// (the host-side name of the array is not a device address).
+reco_status ppl_static_scratch(float **out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 128) return fail(RECO_EUNSUPPORTED, "device index %d out of range", dev);
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_ppl_static_addr[dev]) {
+        float *p = nullptr;
+        e = cudaGetSymbolAddress((void **)&p, g_ppl_static_rows);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(static PPL scratch)");
+        g_ppl_static_addr[dev] = p;
+    }
+    *out = g_ppl_static_addr[dev];
+    return RECO_OK;
+}
+}  // namespace
+
+extern "C" reco_status reco_answer_ppl_static(const float *logits, const int32_t *tokens, const int32_t *n_valid,
+                                              int B, int n, int V, float tau_p, float *ppl, uint8_t *stop,
+                                              cudaStream_t stream)
+{
+    if (B < 1 || n < 0 || V < 1) return fail(RECO_EINVAL, "need B >= 1, n >= 0, V >= 1");
+    if ((long long)B * n > RECO_PPL_STATIC_MAX_ROWS)
+        return fail(RECO_EINVAL, "B*n = %lld answer rows exceed the static scratch of %d rows", (long long)B * n,
+                    RECO_PPL_STATIC_MAX_ROWS);
+    if (!ppl || !stop || (n > 0 && (!logits || !tokens))) return fail(RECO_EINVAL, "NULL logits, tokens, ppl or stop");
+    if (((uintptr_t)logits & 3u)) return fail(RECO_EINVAL, "logits must be 4-byte aligned");
+    float *scratch;
+    reco_status st = ppl_static_scratch(&scratch);
+    if (st != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_ppl(logits, tokens, n_valid, B, n, V, tau_p, ppl, stop, scratch, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_answer_ppl_static launch");
+}

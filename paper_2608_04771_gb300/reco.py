@@ -20,7 +20,9 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL = range(4)
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_answer_ppl")
+           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_answer_ppl",
+           "reco_answer_ppl_static")
+RECO_PPL_STATIC_MAX_ROWS = 65536
 
 
 class RecoError(RuntimeError):
@@ -65,9 +67,10 @@ def lib():
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
+    L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
                  "reco_score_cache", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty",
-                 "reco_answer_ppl"):
+                 "reco_answer_ppl", "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
     _lib = L
     return L
@@ -175,3 +178,10 @@ def reco_answer_ppl(logits, tokens, n_valid, tau_p, ppl, stop, ws, stream=None):
     B, n, V = logits.shape
     _ok(lib().reco_answer_ppl(_ptr(logits), _ptr(tokens), _ptr(n_valid), B, n, V, float(tau_p),
                               _ptr(ppl), _ptr(stop), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_answer_ppl_static(logits, tokens, n_valid, tau_p, ppl, stop, stream=None):
+    """reco_answer_ppl without a workspace: the library's fixed scratch array is used."""
+    B, n, V = logits.shape
+    _ok(lib().reco_answer_ppl_static(_ptr(logits), _ptr(tokens), _ptr(n_valid), B, n, V, float(tau_p),
+                                     _ptr(ppl), _ptr(stop), _stream(stream)))
