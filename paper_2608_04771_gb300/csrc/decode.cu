@@ -63,6 +63,14 @@ struct DecodeArgs {
     unsigned *err;
 };
 
+// atomicAdd with acquire-release semantics at GPU scope.
+__device__ __forceinline__ int atom_add_acq_rel(int *p, int v)
+{
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
 __device__ __forceinline__ bool unit_ok(int L, int L_cap, int append)
 {
     return L >= 0 && L <= L_cap && (!append || L < L_cap);
@@ -204,7 +212,8 @@ __device__ __forceinline__ uint32_t word(const uint4 &v, int x)
 
 constexpr int kDecodeWarps = 8;       // warps per CTA (one CTA per SM)
 constexpr int kDecodeStages = 3;      // ring stages per warp
-constexpr int kMaxTmaUnits = 4096;    // plan entries kept in shared memory
+constexpr int kItemsPerWarp = 4;      // target work items per warp (fewer, larger items pay less per-item cost)
+constexpr int kMaxTmaUnits = 3072;    // two plan entries per unit kept in shared memory
 constexpr long long kSpinLimit = 1LL << 24;  // bounded mbarrier waits (about a second)
 
 template <int D> struct TmaLayout {
@@ -217,7 +226,7 @@ template <int D> struct TmaLayout {
 template <int D>
 size_t tma_smem_bytes(int units)
 {
-    return 1024 + (size_t)TmaLayout<D>::RING + (size_t)(units + 1) * sizeof(int);
+    return 1024 + (size_t)TmaLayout<D>::RING + 2 * (size_t)(units + 1) * sizeof(int);
 }
 
 // Byte offset of 16-byte chunk ch (0..7) of row rr inside a 128B-swizzled 16-row box.
@@ -234,10 +243,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NW][S];
     __shared__ long long sm_red[NW];
-    __shared__ int sm_scan[NW];
+    __shared__ int sm_scan[NW], sm_scan2[NW];
     const uint32_t raw0 = (uint32_t)__cvta_generic_to_shared(smem_raw);
     const uint32_t ring0 = (raw0 + 1023u) & ~1023u;
-    int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
+    int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // 2 x [units + 1]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
     const uint32_t my_ring = ring0 + (uint32_t)wid * S * STAGE;
@@ -248,16 +257,30 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
     __syncwarp();
 
-    // ---- plan: identical in every CTA (lens are not modified until every warp is done)
+    // ---- plan: identical in every CTA (lens are not modified until every warp is done).
+    // Unit u splits into nf_u = le_u / C full chunks and, when le_u % C != 0 (or the unit
+    // is empty), one shorter tail chunk.  Items are handed out full chunks first, tails
+    // last, so the final items are short and the end of the launch drains evenly.
+    int *pre_f = sm_pre;              // [units + 1] prefix of full chunks
+    int *pre_t = sm_pre + units + 1;  // [units + 1] prefix of tail chunks
     const int seg = (units + blockDim.x - 1) / blockDim.x;
     const int u_lo = min(units, tid * seg), u_hi = min(units, u_lo + seg);
-    long long tot = 0;
-    for (int u = u_lo; u < u_hi; ++u) {
+    auto eff_len = [&](int u) {
+        const int L = a.lens[u];
+        return unit_ok(L, a.L_cap, a.append) ? L + a.append : -1;
+    };
+    // stage the lengths in the (still idle) ring memory with one coalesced sweep; the
+    // plan below reads them from there (the ring is first written by TMA after the plan)
+    int *len_sm = reinterpret_cast<int *>(smem_raw + (ring0 - raw0));
+    for (int u = tid; u < units; u += blockDim.x) {
         const int L = a.lens[u];
         const bool ok = unit_ok(L, a.L_cap, a.append);
         if (!ok && blockIdx.x == 0) raise_error(a.err, (a.append && L == a.L_cap) ? ERR_ROOM : ERR_LEN);
-        tot += ok ? L + a.append : 0;
+        len_sm[u] = ok ? L + a.append : 0;
     }
+    __syncthreads();
+    long long tot = 0;
+    for (int u = u_lo; u < u_hi; ++u) tot += len_sm[u];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
     if (lane == 0) sm_red[wid] = tot;
@@ -265,59 +288,161 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     tot = 0;
     for (int w2 = 0; w2 < NW; ++w2) tot += sm_red[w2];
     const int total_warps = gridDim.x * NW;
-    const long long target = min((long long)kDecodeMaxTarget, 8LL * total_warps);
-    long long C = (tot + target - 1) / target;
-    C = ((C + 63) / 64) * 64;
-    if (C < 256) C = 256;
-    auto eff_len = [&](int u) {
-        const int L = a.lens[u];
-        return unit_ok(L, a.L_cap, a.append) ? L + a.append : -1;
-    };
-    int my_items = 0;
-    for (int u = u_lo; u < u_hi; ++u) my_items += max(1, (int)((max(eff_len(u), 0) + C - 1) / C));
+    const long long target = min((long long)kDecodeMaxTarget, (long long)kItemsPerWarp * total_warps);
+    long long Cl = (tot + target - 1) / target;
+    Cl = ((Cl + 63) / 64) * 64;
+    if (Cl < 256) Cl = 256;
+    const int C = (int)Cl;
+    int my_f = 0, my_t = 0;
+    for (int u = u_lo; u < u_hi; ++u) {
+        const int le = len_sm[u];
+        my_f += le / C;
+        my_t += (le % C != 0 || le == 0) ? 1 : 0;
+    }
     {
-        int incl = my_items;
+        int f = my_f, t2 = my_t;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int n = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += n;
+            const int nf = __shfl_up_sync(0xffffffffu, f, o), nt = __shfl_up_sync(0xffffffffu, t2, o);
+            if (lane >= o) {
+                f += nf;
+                t2 += nt;
+            }
         }
-        if (lane == 31) sm_scan[wid] = incl;
+        if (lane == 31) {
+            sm_scan[wid] = f;
+            sm_scan2[wid] = t2;
+        }
         __syncthreads();
-        int run = incl - my_items;
-        for (int w2 = 0; w2 < wid; ++w2) run += sm_scan[w2];
-        for (int u = u_lo; u < u_hi; ++u) {
-            sm_pre[u] = run;
-            run += max(1, (int)((max(eff_len(u), 0) + C - 1) / C));
+        int rf = f - my_f, rt = t2 - my_t;
+        for (int w2 = 0; w2 < wid; ++w2) {
+            rf += sm_scan[w2];
+            rt += sm_scan2[w2];
         }
-        if (tid == blockDim.x - 1) sm_pre[units] = run;
+        for (int u = u_lo; u < u_hi; ++u) {
+            pre_f[u] = rf;
+            pre_t[u] = rt;
+            const int le = len_sm[u];
+            rf += le / C;
+            rt += (le % C != 0 || le == 0) ? 1 : 0;
+        }
+        if (tid == blockDim.x - 1) {
+            pre_f[units] = rf;
+            pre_t[units] = rt;
+        }
     }
     __syncthreads();
-    const int total_items = sm_pre[units];
+    const int NF = pre_f[units];
+    const int total_items = NF + pre_t[units];
     const int g = lane >> 2, c = lane & 3;
     const bool out_bf16 = a.out_bf16 != 0;
-    uint32_t gblk = 0;  // 16-key blocks this warp has pushed through its ring
-    bool aborted = false;
 
-    for (;;) {
-        int item = 0;
-        if (lane == 0) item = atomicAdd(&a.counters[0], 1);
-        item = __shfl_sync(0xffffffffu, item, 0);
-        if (item >= total_items) break;
-        int lo = 0, hi = units - 1;  // last unit whose first item <= item
+    // dispatch index -> (unit, chunk) and the chunk's key range
+    struct Item {
+        int u, split, first, nsplit, le, k0, k1, Lapp, nblk;
+    };
+    auto last_le = [](const int *pre, int units_, int d) {  // largest u with pre[u] <= d
+        int lo = 0, hi = units_ - 1;
         while (lo < hi) {
             const int mid = (lo + hi + 1) >> 1;
-            if (sm_pre[mid] <= item) lo = mid; else hi = mid - 1;
+            if (pre[mid] <= d) lo = mid; else hi = mid - 1;
         }
-        const int u = lo;
-        const int first = sm_pre[u], nsplit = sm_pre[u + 1] - first;
-        const int split = item - first;
+        return lo;
+    };
+    auto meta = [&](int d) {
+        Item it;
+        it.nblk = -1;  // no item
+        if (d >= total_items) return it;
+        int u, split;
+        if (d < NF) {
+            u = last_le(pre_f, units, d);
+            split = d - pre_f[u];
+        } else {
+            u = last_le(pre_t, units, d - NF);
+            split = pre_f[u + 1] - pre_f[u];
+        }
         const int le_raw = eff_len(u);
-        const bool valid = le_raw >= 0;
-        const int le = valid ? le_raw : 0;
-        const int Lapp = (valid && a.append) ? le - 1 : -1;  // index of the appended row
-        const int k0 = (int)min((long long)split * C, (long long)le);
-        const int k1 = (int)min((long long)k0 + C, (long long)le);
+        it.u = u;
+        it.split = split;
+        it.first = pre_f[u] + pre_t[u];
+        it.nsplit = (pre_f[u + 1] - pre_f[u]) + (pre_t[u + 1] - pre_t[u]);
+        it.le = le_raw >= 0 ? le_raw : 0;
+        it.Lapp = (le_raw >= 0 && a.append) ? it.le - 1 : -1;
+        it.k0 = min(split * C, it.le);
+        it.k1 = min(it.k0 + C, it.le);
+        it.nblk = (it.k1 - it.k0 + 15) / 16;
+        return it;
+    };
+    auto grab = [&]() {
+        int d = 0;
+        if (lane == 0) d = atomicAdd(&a.counters[0], 1);
+        d = __shfl_sync(0xffffffffu, d, 0);
+        return meta(d);
+    };
+
+    // Q fragments of an item (rows g < G), head dim permuted to match the K chunks:
+    // k-step j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
+    // and + {2,3} (a2).
+    auto load_q = [&](const Item &it, uint32_t (&qa)[D / 16][2]) {
+        const long qrow = (long)(it.u / a.Hkv) * a.Hq + (long)(it.u % a.Hkv) * a.G;
+        const __nv_bfloat16 *qp = reinterpret_cast<const __nv_bfloat16 *>(a.q) + (qrow + g) * D;
+#pragma unroll
+        for (int hh = 0; hh < HALVES; ++hh)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                uint4 wv = make_uint4(0, 0, 0, 0);
+                if (g < a.G) wv = *reinterpret_cast<const uint4 *>(qp + 64 * hh + 16 * c + 8 * e);
+                const int j = 4 * hh + 2 * e;
+                qa[j][0] = wv.x;
+                qa[j][1] = wv.y;
+                qa[j + 1][0] = wv.z;
+                qa[j + 1][1] = wv.w;
+            }
+    };
+
+    // ---- block stream: lane 0 keeps up to S blocks in flight, running from the current
+    // item into the next one (grabbed one item ahead) so no refill bubble opens between
+    // items; the warp consumes blocks in issue order.
+    uint32_t issued = 0, consumed = 0;
+    Item cur = grab();
+    Item nxt = cur.nblk >= 0 ? grab() : cur;
+    uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
+    if (cur.nblk >= 0) load_q(cur, qa_n);
+    Item pit = cur;  // item the producer is issuing from
+    int pblk = 0;
+    bool p_on_next = false;
+    bool aborted = false;
+    auto can_issue = [&]() {
+        if (pblk < pit.nblk) return true;
+        if (!p_on_next && nxt.nblk > 0) {
+            pit = nxt;
+            pblk = 0;
+            p_on_next = true;
+            return true;
+        }
+        return false;
+    };
+    auto issue = [&]() {
+        const uint32_t slot = issued % S;
+        if (lane == 0) {
+            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
+            const uint32_t dst = my_ring + slot * STAGE;
+            const int y = pit.u * a.L_cap + pit.k0 + 16 * pblk;
+            fence_async_shared();
+            mbar_expect_tx(bar, STAGE);
+#pragma unroll
+            for (int hh = 0; hh < HALVES; ++hh) {
+                tma_load_2d(dst + hh * TILE, &tmK, 64 * hh, y, bar);
+                tma_load_2d(dst + (HALVES + hh) * TILE, &tmV, 64 * hh, y, bar);
+            }
+        }
+        ++pblk;
+        ++issued;
+    };
+
+    while (cur.nblk >= 0) {
+        const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
+        const int first = cur.first, nsplit = cur.nsplit, item = first + cur.split;  // partial slot
         const long lb = u / a.Hkv;
         const int h = u % a.Hkv;
         const int G = a.G;
@@ -326,65 +451,29 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         const long qrow0 = lb * a.Hq + (long)h * G;
         const int row0 = u * a.L_cap;  // first tensor-map row of this unit
 
-        // Q fragments (rows g < G), head dim permuted to match the K chunks: k-step
-        // j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
-        // and + {2,3} (a2).
         uint32_t qa[D / 16][2];
-        {
-            const __nv_bfloat16 *qp = reinterpret_cast<const __nv_bfloat16 *>(a.q) + (qrow0 + g) * D;
 #pragma unroll
-            for (int hh = 0; hh < HALVES; ++hh)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    uint4 wv = make_uint4(0, 0, 0, 0);
-                    if (g < G) wv = *reinterpret_cast<const uint4 *>(qp + 64 * hh + 16 * c + 8 * e);
-                    const int j = 4 * hh + 2 * e;
-                    qa[j][0] = wv.x;
-                    qa[j][1] = wv.y;
-                    qa[j + 1][0] = wv.z;
-                    qa[j + 1][1] = wv.w;
-                }
+        for (int j = 0; j < D / 16; ++j) {
+            qa[j][0] = qa_n[j][0];
+            qa[j][1] = qa_n[j][1];
         }
+        if (nxt.nblk >= 0) load_q(nxt, qa_n);  // the next item's queries load while this one streams
         float o[MT][4];
 #pragma unroll
         for (int t = 0; t < MT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
         float m = -INFINITY, l = 0.f;
 
-        const int nblk = (k1 - k0 + 15) / 16;
-        const uint32_t blk0 = gblk;
-        auto issue = [&](int bi) {  // lane 0 only
-            const uint32_t slot = (blk0 + bi) % S;
-            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
-            const uint32_t dst = my_ring + slot * STAGE;
-            const int y = row0 + k0 + 16 * bi;
-            fence_async_shared();
-            mbar_expect_tx(bar, STAGE);
-#pragma unroll
-            for (int hh = 0; hh < HALVES; ++hh) {
-                tma_load_2d(dst + hh * TILE, &tmK, 64 * hh, y, bar);
-                tma_load_2d(dst + (HALVES + hh) * TILE, &tmV, 64 * hh, y, bar);
-            }
-        };
-        if (lane == 0)
-            for (int p = 0; p < S - 1 && p < nblk; ++p) issue(p);
-        for (int bi = 0; bi < nblk; ++bi) {
+        for (int bi = 0; bi < cur.nblk; ++bi) {
             __syncwarp();
-            if (lane == 0 && bi + S - 1 < nblk) issue(bi + S - 1);
-            const uint32_t slot = (blk0 + bi) % S;
-            const uint32_t parity = ((blk0 + bi) / S) & 1u;
+            while (issued - consumed < (uint32_t)S && can_issue()) issue();
+            const uint32_t slot = consumed % S;
+            const uint32_t parity = (consumed / S) & 1u;
             const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
-            long long spins = 0;
-            while (!mbar_try_wait(bar, parity)) {
-                if (++spins > kSpinLimit) break;
-            }
-            if (spins > kSpinLimit) {  // a copy never landed: report, drain what is in flight, stop
+            if (!mbar_wait_bounded(bar, parity, kSpinLimit)) {  // a copy never landed: report, drain, stop
                 if (lane == 0) raise_error(a.err, ERR_INTERNAL);
-                for (int p = bi + 1; p < nblk && p < bi + S; ++p) {
-                    const uint32_t sl = (blk0 + p) % S, par = ((blk0 + p) / S) & 1u;
-                    const uint32_t b2 = (uint32_t)__cvta_generic_to_shared(&bars[wid][sl]);
-                    for (long long t2 = 0; t2 < kSpinLimit && !mbar_try_wait(b2, par); ++t2) {
-                    }
-                }
+                for (uint32_t q2 = consumed + 1; q2 < issued; ++q2)
+                    mbar_wait_bounded((uint32_t)__cvta_generic_to_shared(&bars[wid][q2 % S]), (q2 / S) & 1u,
+                                      kSpinLimit);
                 aborted = true;
                 break;
             }
@@ -465,9 +554,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                     mma_bf16(o[4 * hh + x], A0, A1, A2, A3, pl0, pl1);
                 }
             }
+            ++consumed;
         }
-        gblk += nblk;
         if (aborted) break;
+
         l += __shfl_xor_sync(0xffffffffu, l, 1);
         l += __shfl_xor_sync(0xffffffffu, l, 2);
 
@@ -519,47 +609,93 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 a.part_ml[((size_t)item * G + g) * 2 + 0] = m;
                 a.part_ml[((size_t)item * G + g) * 2 + 1] = l;
             }
-            __threadfence();
+            // publish: the warp barrier orders every lane's partial writes before lane 0's
+            // release; the last arriver's acquire (and the barrier after it) orders its reads
             __syncwarp();
             int old = 0;
-            if (lane == 0) old = atomicAdd(&a.counters[2 + u], 1);
+            if (lane == 0) old = atom_add_acq_rel(&a.counters[2 + u], 1);
             old = __shfl_sync(0xffffffffu, old, 0);
+            __syncwarp();
             if (old == nsplit - 1) {  // last item of this unit: merge the partials
-                __threadfence();
+                // pass 1: per-query-head maxima, lanes over splits (independent loads)
+                float Mq[8];
+#pragma unroll
+                for (int qq = 0; qq < 8; ++qq) Mq[qq] = -INFINITY;
+                for (int sb = 0; sb < nsplit; sb += 32) {
+                    const int s2 = sb + lane;
+                    if (s2 < nsplit) {
+#pragma unroll
+                        for (int qq = 0; qq < 8; ++qq)
+                            if (qq < G) Mq[qq] = fmaxf(Mq[qq], __ldcg(a.part_ml + ((size_t)(first + s2) * G + qq) * 2));
+                    }
+                }
+#pragma unroll
+                for (int qq = 0; qq < 8; ++qq) Mq[qq] = warp_max(Mq[qq]);
+                // pass 2: every lane owns 4 head-dim elements of all G heads; one sweep over
+                // the splits with all of a split's loads issued together
                 constexpr int PER = D / 32;
-                for (int qq = 0; qq < G; ++qq) {
-                    float M = -INFINITY;
-                    for (int s2 = 0; s2 < nsplit; ++s2)
-                        M = fmaxf(M, __ldcg(a.part_ml + ((size_t)(first + s2) * G + qq) * 2));
-                    float Ls = 0.f, acc[PER];
+                float acc[8][PER], Lq[8];
 #pragma unroll
-                    for (int e = 0; e < PER; ++e) acc[e] = 0.f;
-                    if (M != -INFINITY) {
-                        for (int s2 = 0; s2 < nsplit; ++s2) {
-                            const size_t it = (size_t)(first + s2) * G + qq;
-                            const float wt = fast_exp2(__ldcg(a.part_ml + it * 2) - M);
-                            Ls += __ldcg(a.part_ml + it * 2 + 1) * wt;
-                            const float *src = a.part_o + it * D + lane * PER;
+                for (int qq = 0; qq < 8; ++qq) {
+                    Lq[qq] = 0.f;
 #pragma unroll
-                            for (int e = 0; e < PER; ++e) acc[e] += __ldcg(src + e) * wt;
+                    for (int e = 0; e < PER; ++e) acc[qq][e] = 0.f;
+                }
+#pragma unroll 2
+                for (int s2 = 0; s2 < nsplit; ++s2) {
+                    const size_t it0 = (size_t)(first + s2) * G;
+#pragma unroll
+                    for (int qq = 0; qq < 8; ++qq) {
+                        if (qq < G && Mq[qq] != -INFINITY) {
+                            const float2 ml = __ldcg(reinterpret_cast<const float2 *>(a.part_ml) + it0 + qq);
+                            const float wt = fast_exp2(ml.x - Mq[qq]);
+                            Lq[qq] += ml.y * wt;
+                            const float *src = a.part_o + (it0 + qq) * D + lane * PER;
+                            if constexpr (PER == 4) {
+                                const float4 ov = __ldcg(reinterpret_cast<const float4 *>(src));
+                                acc[qq][0] += ov.x * wt;
+                                acc[qq][1] += ov.y * wt;
+                                acc[qq][2] += ov.z * wt;
+                                acc[qq][3] += ov.w * wt;
+                            } else {
+#pragma unroll
+                                for (int e = 0; e < PER; ++e) acc[qq][e] += __ldcg(src + e) * wt;
+                            }
                         }
                     }
-                    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+                }
 #pragma unroll
-                    for (int e = 0; e < PER; ++e)
-                        store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + qq) * D + lane * PER + e, acc[e] * inv);
-                    if (lane == 0 && a.lse) a.lse[qrow0 + qq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+                for (int qq = 0; qq < 8; ++qq) {
+                    if (qq < G) {
+                        const float inv = Lq[qq] > 0.f ? 1.f / Lq[qq] : 0.f;
+#pragma unroll
+                        for (int e = 0; e < PER; ++e)
+                            store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + qq) * D + lane * PER + e,
+                                                     acc[qq][e] * inv);
+                        if (lane == 0 && a.lse)
+                            a.lse[qrow0 + qq] = Lq[qq] > 0.f ? (Mq[qq] + log2f(Lq[qq])) * kLn2 : -INFINITY;
+                    }
                 }
             }
+        }
+        // advance: the producer may already be streaming the next item's blocks
+        cur = nxt;
+        nxt = cur.nblk >= 0 ? grab() : cur;
+        if (p_on_next) {
+            p_on_next = false;
+        } else {
+            pit = cur;
+            pblk = 0;
         }
     }
     if (aborted) return;
     // the last warp of the grid advances the lengths (every plan has been read by then)
     int done = 0;
-    if (lane == 0) done = atomicAdd(&a.counters[1], 1);
+    __syncwarp();
+    if (lane == 0) done = atom_add_acq_rel(&a.counters[1], 1);
     done = __shfl_sync(0xffffffffu, done, 0);
+    __syncwarp();
     if (done == total_warps - 1 && a.append) {
-        __threadfence();
         for (int u = lane; u < units; u += 32) {
             const int le = eff_len(u);
             if (le >= 0) a.lens[u] = le;

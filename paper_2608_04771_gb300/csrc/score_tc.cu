@@ -1,6 +1,7 @@
 // score_tc.cu -- tensor-core (tcgen05) passes of the Eq. 2 cache scores for bf16 caches.
 //
-// Both passes run one CTA per (unit, 2048-key chunk) with the same roles:
+// Both passes are persistent (one CTA per SM walking a contiguous range of (unit,
+// 2048-key chunk) items, barrier phases running on across items) with the same roles:
 //   warp 0  lane 0 : TMA producer (window queries once, then a ring of K tiles)
 //   warp 1         : allocates 512 TMEM columns; lane 0 issues tcgen05.mma (bf16 in,
 //                    fp32 accumulate in TMEM) and commits to mbarriers
@@ -91,6 +92,7 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
 }
 
 constexpr long long kTcSpin = 1LL << 24;
+constexpr int kTcMaxR = 384;  // window rows (G*w) the tensor-core passes take; pass 2 smem stays < 227 KB
 constexpr int kTmemCols = 512;
 
 __device__ __forceinline__ bool wait_or_flag(uint32_t bar, uint32_t parity, volatile int *abort_flag,
@@ -105,12 +107,36 @@ __device__ __forceinline__ bool wait_or_flag(uint32_t bar, uint32_t parity, vola
     return false;
 }
 
+// ---------------------------------------------------------------- work items
+// A CTA walks a contiguous range of (unit, 2048-key chunk) items in unit order, so its
+// window queries change only when the unit does.
+struct ChunkItem {
+    long u;
+    int chunk, L, j0, j1, ntiles;
+    bool valid;  // the unit's length is in range
+};
+
+__device__ __forceinline__ ChunkItem chunk_item(int i, int n_chunks, const int32_t *lens, int w, int L_cap,
+                                               bool candidates_only, int tile)
+{
+    ChunkItem it;
+    it.u = i / n_chunks;
+    it.chunk = i % n_chunks;
+    it.L = lens[it.u];
+    it.valid = it.L >= w && it.L <= L_cap;
+    const int end = it.valid ? (candidates_only ? it.L - w : it.L) : 0;
+    it.j0 = it.chunk * kScoreChunk;
+    it.j1 = min(it.j0 + kScoreChunk, end);
+    it.ntiles = it.j0 < it.j1 ? (it.j1 - it.j0 + tile - 1) / tile : 0;
+    return it;
+}
+
 // ---------------------------------------------------------------- pass 1: row statistics
 template <int D, int N, int MT>
 __global__ void __launch_bounds__(128 + 128 * MT, 1)
     score_rowstats_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R,
-                      int n_chunks, float c2, float *__restrict__ part_m, float *__restrict__ part_z,
+                      int n_chunks, int n_items, float c2, float *__restrict__ part_m, float *__restrict__ part_z,
                       unsigned *err)
 {
     constexpr int HALVES = D / 64;
@@ -120,34 +146,21 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
     constexpr int NS = 4;
     constexpr uint32_t IDESC = idesc_bf16(128, N);
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    __shared__ __align__(8) uint64_t bar_q, bar_kfull[NS], bar_kempty[NS], bar_afull[2], bar_aempty[2];
+    __shared__ __align__(8) uint64_t bar_qfull, bar_qempty, bar_kfull[NS], bar_kempty[NS], bar_afull[2],
+        bar_aempty[2];
     __shared__ uint32_t tmem_sh;
     __shared__ int abort_sh;
 
-    const int chunk = blockIdx.x;
-    const long u = blockIdx.y;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int L = lens[u];
-    if (L < w || L > L_cap) {
-        if (chunk == 0 && tid == 0) raise_error(err, ERR_LEN);
-        return;
-    }
-    const int j0 = chunk * kScoreChunk;
-    const int j1 = min(j0 + kScoreChunk, L);
-    const int ntiles = j0 < j1 ? (j1 - j0 + N - 1) / N : 0;
-    if (ntiles == 0) {  // chunk past the end: empty statistics
-        for (int r = tid; r < R; r += blockDim.x) {
-            part_m[((size_t)u * n_chunks + chunk) * R + r] = -INFINITY;
-            part_z[((size_t)u * n_chunks + chunk) * R + r] = 0.f;
-        }
-        return;
-    }
+    const int i_begin = (int)((long long)blockIdx.x * n_items / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_items / gridDim.x);
     const uint32_t raw0 = smem_addr(smem_raw);
     const uint32_t base = (raw0 + 1023u) & ~1023u;
     const uint32_t Qs = base;                                  // MT x HALVES x QBOX
     const uint32_t Ks = base + (uint32_t)MT * HALVES * QBOX;  // NS x KSTAGE
     if (tid == 0) {
-        mbar_init(smem_addr(&bar_q), 1);
+        mbar_init(smem_addr(&bar_qfull), 1);
+        mbar_init(smem_addr(&bar_qempty), 1);
         for (int s = 0; s < NS; ++s) {
             mbar_init(smem_addr(&bar_kfull[s]), 1);
             mbar_init(smem_addr(&bar_kempty[s]), 1);
@@ -167,89 +180,129 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
-    const long lb = u / Hkv;
-    const int h = (int)(u % Hkv);
-    const int q_row0 = (int)((lb * Hq + (long)h * G) * w);
-    const int k_row0 = (int)(u * L_cap + j0);
     volatile int *abort_flag = &abort_sh;
 
     if (warp == 0) {
-        if (lane == 0) {  // producer
-            mbar_expect_tx(smem_addr(&bar_q), (uint32_t)MT * HALVES * QBOX);
-            for (int mt = 0; mt < MT; ++mt)
-                for (int hh = 0; hh < HALVES; ++hh)
-                    tma_load_2d(Qs + (mt * HALVES + hh) * QBOX, &tmQ, 64 * hh, q_row0 + 128 * mt, smem_addr(&bar_q));
-            for (int t = 0; t < ntiles; ++t) {
-                const int s = t % NS;
-                const uint32_t ph = (t / NS) & 1;
-                if (!wait_or_flag(smem_addr(&bar_kempty[s]), ph ^ 1, abort_flag, err)) break;
-                mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
-                for (int hh = 0; hh < HALVES; ++hh)
-                    tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * N, smem_addr(&bar_kfull[s]));
+        if (lane == 0) {  // producer: queries when the unit changes, then the chunk's K tiles
+            int gt = 0, nq = 0;
+            long prev_u = -1;
+            bool ok = true;
+            for (int i = i_begin; ok && i < i_end; ++i) {
+                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+                if (it.ntiles == 0) continue;
+                if (it.u != prev_u) {
+                    if (nq > 0 && !wait_or_flag(smem_addr(&bar_qempty), (nq - 1) & 1, abort_flag, err)) break;
+                    const long lb = it.u / Hkv;
+                    const int q_row0 = (int)((lb * Hq + (it.u % Hkv) * G) * w);
+                    mbar_expect_tx(smem_addr(&bar_qfull), (uint32_t)MT * HALVES * QBOX);
+                    for (int mt = 0; mt < MT; ++mt)
+                        for (int hh = 0; hh < HALVES; ++hh)
+                            tma_load_2d(Qs + (mt * HALVES + hh) * QBOX, &tmQ, 64 * hh, q_row0 + 128 * mt,
+                                        smem_addr(&bar_qfull));
+                    ++nq;
+                    prev_u = it.u;
+                }
+                const int k_row0 = (int)(it.u * L_cap + it.j0);
+                for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                    const int s = gt % NS;
+                    if (!wait_or_flag(smem_addr(&bar_kempty[s]), ((gt / NS) & 1) ^ 1, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
+                    for (int hh = 0; hh < HALVES; ++hh)
+                        tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * N, smem_addr(&bar_kfull[s]));
+                }
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {  // MMA issuer
-            bool ok = wait_or_flag(smem_addr(&bar_q), 0, abort_flag, err);
-            for (int t = 0; ok && t < ntiles; ++t) {
-                const int s = t % NS, b = t & 1;
-                const uint32_t ph = (t / NS) & 1, bph = (t >> 1) & 1;
-                if (!wait_or_flag(smem_addr(&bar_kfull[s]), ph, abort_flag, err)) break;
-                if (!wait_or_flag(smem_addr(&bar_aempty[b]), bph ^ 1, abort_flag, err)) break;
-                tc_fence_after();
-                for (int mt = 0; mt < MT; ++mt) {
-                    const uint32_t d = tmem + (uint32_t)((b * MT + mt) * N);
-#pragma unroll
-                    for (int k = 0; k < D / 16; ++k) {
-                        const int hh = k >> 2, kk = k & 3;
-                        const uint64_t ad = sw128_desc(Qs + (mt * HALVES + hh) * QBOX + kk * 32);
-                        const uint64_t bd = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
-                        tc_mma(d, ad, bd, IDESC, k > 0 ? 1u : 0u);
-                    }
+            int gt = 0, nq = 0;
+            long prev_u = -1;
+            bool ok = true;
+            for (int i = i_begin; ok && i < i_end; ++i) {
+                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+                if (it.ntiles == 0) continue;
+                if (it.u != prev_u) {
+                    if (nq > 0) tc_commit(smem_addr(&bar_qempty));  // queries free once prior MMAs land
+                    if (!wait_or_flag(smem_addr(&bar_qfull), nq & 1, abort_flag, err)) break;
+                    ++nq;
+                    prev_u = it.u;
                 }
-                tc_commit(smem_addr(&bar_kempty[s]));
-                tc_commit(smem_addr(&bar_afull[b]));
+                for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                    const int s = gt % NS, b = gt & 1;
+                    if (!wait_or_flag(smem_addr(&bar_kfull[s]), (gt / NS) & 1, abort_flag, err) ||
+                        !wait_or_flag(smem_addr(&bar_aempty[b]), ((gt >> 1) & 1) ^ 1, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int mt = 0; mt < MT; ++mt) {
+                        const uint32_t d = tmem + (uint32_t)((b * MT + mt) * N);
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k) {
+                            const int hh = k >> 2, kk = k & 3;
+                            const uint64_t ad = sw128_desc(Qs + (mt * HALVES + hh) * QBOX + kk * 32);
+                            const uint64_t bd = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
+                            tc_mma(d, ad, bd, IDESC, k > 0 ? 1u : 0u);
+                        }
+                    }
+                    tc_commit(smem_addr(&bar_kempty[s]));
+                    tc_commit(smem_addr(&bar_afull[b]));
+                }
             }
         }
     } else if (warp >= 4 && warp < 4 + 4 * MT) {  // epilogue: one window row per thread
         const int e = warp - 4, mt = e >> 2, quarter = warp & 3;
         const int r = mt * 128 + quarter * 32 + lane;
         const int t_row = r % w;
-        const int jmax = L - w + t_row;  // last key this window row sees
-        float m = -INFINITY, z = 0.f;
-        for (int t = 0; t < ntiles; ++t) {
-            const int b = t & 1;
-            const uint32_t bph = (t >> 1) & 1;
-            if (!wait_or_flag(smem_addr(&bar_afull[b]), bph, abort_flag, err)) break;
-            tc_fence_after();
-            const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((b * MT + mt) * N);
-            const int jb = j0 + t * N;
-            const int lim = min(j1 - 1, jmax) - jb;  // columns 0..lim are visible to this row
-#pragma unroll 1
-            for (int cc = 0; cc < N; cc += 32) {
-                float v[32];
-                tmem_ld32(ta + cc, v);
-                float mx = -INFINITY;
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    v[i] *= c2;
-                    if (cc + i <= lim) mx = fmaxf(mx, v[i]);
-                }
-                const float mn = fmaxf(m, mx);
-                if (mn == -INFINITY) continue;
-                float acc = 0.f;
-#pragma unroll
-                for (int i = 0; i < 32; ++i) acc += (cc + i <= lim) ? fast_exp2(v[i] - mn) : 0.f;
-                z = z * fast_exp2(m - mn) + acc;
-                m = mn;
+        int gt = 0;
+        for (int i = i_begin; i < i_end; ++i) {
+            const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+            if (!it.valid) {
+                if (it.chunk == 0 && r == 0) raise_error(err, ERR_LEN);
+                continue;
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
-        }
-        if (r < R && !*abort_flag) {
-            part_m[((size_t)u * n_chunks + chunk) * R + r] = m;
-            part_z[((size_t)u * n_chunks + chunk) * R + r] = z;
+            const int jmax = it.L - w + t_row;  // last key this window row sees
+            float m = -INFINITY, z = 0.f;
+            bool ok = true;
+            for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                const int b = gt & 1;
+                if (!wait_or_flag(smem_addr(&bar_afull[b]), (gt >> 1) & 1, abort_flag, err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((b * MT + mt) * N);
+                const int jb = it.j0 + t * N;
+                const int lim = min(it.j1 - 1, jmax) - jb;  // columns 0..lim are visible to this row
+#pragma unroll 1
+                for (int cc = 0; cc < N; cc += 32) {
+                    float v[32];
+                    tmem_ld32(ta + cc, v);
+                    float mx = -INFINITY;
+#pragma unroll
+                    for (int q = 0; q < 32; ++q) {
+                        v[q] *= c2;
+                        if (cc + q <= lim) mx = fmaxf(mx, v[q]);
+                    }
+                    const float mn = fmaxf(m, mx);
+                    if (mn == -INFINITY) continue;
+                    float acc = 0.f;
+#pragma unroll
+                    for (int q = 0; q < 32; ++q) acc += (cc + q <= lim) ? fast_exp2(v[q] - mn) : 0.f;
+                    z = z * fast_exp2(m - mn) + acc;
+                    m = mn;
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
+            }
+            if (!ok) break;
+            if (r < R) {
+                part_m[((size_t)it.u * n_chunks + it.chunk) * R + r] = m;
+                part_z[((size_t)it.u * n_chunks + it.chunk) * R + r] = z;
+            }
         }
     }
     __syncthreads();
@@ -260,35 +313,30 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
 }
 
 // ---------------------------------------------------------------- pass 2: column sums
-// NQ (runtime, multiple of 16, <= 512) query columns per tile.  With NQ <= 256 the two
+// NQ (runtime, multiple of 16, <= 384) query columns per tile.  With NQ <= 256 the two
 // epilogue warpgroups take alternate tiles (two TMEM buffers); above 256 one buffer is
 // shared and each warpgroup sums half of the columns.
 template <int D>
 __global__ void __launch_bounds__(128 + 256, 1)
     score_colsum_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R, int NQ,
-                    float c2, const float *__restrict__ rowb, float *__restrict__ raw, unsigned *err)
+                    int n_chunks, int n_items, float c2, const float *__restrict__ rowb, float *__restrict__ raw,
+                    unsigned *err)
 {
     constexpr int HALVES = D / 64;
     constexpr int KBOX = 128 * 128;  // 128 keys x 128 bytes
     constexpr int KSTAGE = HALVES * KBOX;
     constexpr int NS = 3;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    __shared__ __align__(8) uint64_t bar_q, bar_kfull[NS], bar_kempty[NS], bar_afull[2], bar_aempty[2];
+    __shared__ __align__(8) uint64_t bar_qfull, bar_qempty, bar_kfull[NS], bar_kempty[NS], bar_afull[2],
+        bar_aempty[2];
     __shared__ uint32_t tmem_sh;
     __shared__ int abort_sh;
-    __shared__ float bsh[512];
+    __shared__ float bsh[8][kTcMaxR];  // per epilogue warp: row normalisers of its current unit
 
-    const int chunk = blockIdx.x;
-    const long u = blockIdx.y;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int L = lens[u];
-    if (L < w || L > L_cap) return;
-    const int nc = L - w;
-    const int j0 = chunk * kScoreChunk;
-    const int j1 = min(j0 + kScoreChunk, nc);
-    if (j0 >= j1) return;
-    const int ntiles = (j1 - j0 + 127) / 128;
+    const int i_begin = (int)((long long)blockIdx.x * n_items / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_items / gridDim.x);
     const bool split_cols = NQ > 256;
     const int NBUF = split_cols ? 1 : 2;
     const int nmma = split_cols ? 2 : 1;
@@ -299,9 +347,9 @@ __global__ void __launch_bounds__(128 + 256, 1)
     const uint32_t QBOXB = (uint32_t)NQ * 128;  // one half (64 columns) of all NQ query rows
     const uint32_t Qs = base;
     const uint32_t Ks = base + HALVES * QBOXB;
-    for (int r = tid; r < 512; r += blockDim.x) bsh[r] = r < R ? rowb[u * R + r] : 0.f;
     if (tid == 0) {
-        mbar_init(smem_addr(&bar_q), 1);
+        mbar_init(smem_addr(&bar_qfull), 1);
+        mbar_init(smem_addr(&bar_qempty), 1);
         for (int s = 0; s < NS; ++s) {
             mbar_init(smem_addr(&bar_kfull[s]), 1);
             mbar_init(smem_addr(&bar_kempty[s]), 1);
@@ -321,48 +369,77 @@ __global__ void __launch_bounds__(128 + 256, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
-    const long lb = u / Hkv;
-    const int h = (int)(u % Hkv);
-    const int q_row0 = (int)((lb * Hq + (long)h * G) * w);
-    const int k_row0 = (int)(u * L_cap + j0);
     volatile int *abort_flag = &abort_sh;
 
     if (warp == 0) {
-        if (lane == 0) {
+        if (lane == 0) {  // producer
             const int qbox_rows = NQ > 256 ? NQ / 2 : NQ;
-            mbar_expect_tx(smem_addr(&bar_q), HALVES * QBOXB);
-            for (int hh = 0; hh < HALVES; ++hh)
-                for (int r0 = 0; r0 < NQ; r0 += qbox_rows)
-                    tma_load_2d(Qs + hh * QBOXB + r0 * 128, &tmQ, 64 * hh, q_row0 + r0, smem_addr(&bar_q));
-            for (int t = 0; t < ntiles; ++t) {
-                const int s = t % NS;
-                const uint32_t ph = (t / NS) & 1;
-                if (!wait_or_flag(smem_addr(&bar_kempty[s]), ph ^ 1, abort_flag, err)) break;
-                mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
-                for (int hh = 0; hh < HALVES; ++hh)
-                    tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * 128, smem_addr(&bar_kfull[s]));
+            int gt = 0, nq = 0;
+            long prev_u = -1;
+            bool ok = true;
+            for (int i = i_begin; ok && i < i_end; ++i) {
+                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+                if (it.ntiles == 0) continue;
+                if (it.u != prev_u) {
+                    if (nq > 0 && !wait_or_flag(smem_addr(&bar_qempty), (nq - 1) & 1, abort_flag, err)) break;
+                    const long lb = it.u / Hkv;
+                    const int q_row0 = (int)((lb * Hq + (it.u % Hkv) * G) * w);
+                    mbar_expect_tx(smem_addr(&bar_qfull), HALVES * QBOXB);
+                    for (int hh = 0; hh < HALVES; ++hh)
+                        for (int r0 = 0; r0 < NQ; r0 += qbox_rows)
+                            tma_load_2d(Qs + hh * QBOXB + r0 * 128, &tmQ, 64 * hh, q_row0 + r0, smem_addr(&bar_qfull));
+                    ++nq;
+                    prev_u = it.u;
+                }
+                const int k_row0 = (int)(it.u * L_cap + it.j0);
+                for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                    const int s = gt % NS;
+                    if (!wait_or_flag(smem_addr(&bar_kempty[s]), ((gt / NS) & 1) ^ 1, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(smem_addr(&bar_kfull[s]), KSTAGE);
+                    for (int hh = 0; hh < HALVES; ++hh)
+                        tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * 128,
+                                    smem_addr(&bar_kfull[s]));
+                }
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            bool ok = wait_or_flag(smem_addr(&bar_q), 0, abort_flag, err);
-            for (int t = 0; ok && t < ntiles; ++t) {
-                const int s = t % NS, b = NBUF == 2 ? (t & 1) : 0;
-                const uint32_t ph = (t / NS) & 1, bph = NBUF == 2 ? ((t >> 1) & 1) : (t & 1);
-                if (!wait_or_flag(smem_addr(&bar_kfull[s]), ph, abort_flag, err)) break;
-                if (!wait_or_flag(smem_addr(&bar_aempty[b]), bph ^ 1, abort_flag, err)) break;
-                tc_fence_after();
-                for (int nb = 0; nb < nmma; ++nb) {
-                    const uint32_t d = tmem + (uint32_t)(b * 256 + nb * NM);
-                    for (int k = 0; k < D / 16; ++k) {
-                        const int hh = k >> 2, kk = k & 3;
-                        const uint64_t ad = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
-                        const uint64_t bd = sw128_desc(Qs + hh * QBOXB + nb * NM * 128 + kk * 32);
-                        tc_mma(d, ad, bd, idesc, k > 0 ? 1u : 0u);
-                    }
+        if (lane == 0) {  // MMA issuer
+            int gt = 0, nq = 0;
+            long prev_u = -1;
+            bool ok = true;
+            for (int i = i_begin; ok && i < i_end; ++i) {
+                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+                if (it.ntiles == 0) continue;
+                if (it.u != prev_u) {
+                    if (nq > 0) tc_commit(smem_addr(&bar_qempty));
+                    if (!wait_or_flag(smem_addr(&bar_qfull), nq & 1, abort_flag, err)) break;
+                    ++nq;
+                    prev_u = it.u;
                 }
-                tc_commit(smem_addr(&bar_kempty[s]));
-                tc_commit(smem_addr(&bar_afull[b]));
+                for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                    const int s = gt % NS, b = NBUF == 2 ? (gt & 1) : 0;
+                    const uint32_t bph = NBUF == 2 ? ((gt >> 1) & 1) : (gt & 1);
+                    if (!wait_or_flag(smem_addr(&bar_kfull[s]), (gt / NS) & 1, abort_flag, err) ||
+                        !wait_or_flag(smem_addr(&bar_aempty[b]), bph ^ 1, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int nb = 0; nb < nmma; ++nb) {
+                        const uint32_t d = tmem + (uint32_t)(b * 256 + nb * NM);
+                        for (int k = 0; k < D / 16; ++k) {
+                            const int hh = k >> 2, kk = k & 3;
+                            const uint64_t ad = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
+                            const uint64_t bd = sw128_desc(Qs + hh * QBOXB + nb * NM * 128 + kk * 32);
+                            tc_mma(d, ad, bd, idesc, k > 0 ? 1u : 0u);
+                        }
+                    }
+                    tc_commit(smem_addr(&bar_kempty[s]));
+                    tc_commit(smem_addr(&bar_afull[b]));
+                }
             }
         }
     } else if (warp >= 4) {  // epilogue: one key per thread
@@ -371,30 +448,50 @@ __global__ void __launch_bounds__(128 + 256, 1)
         const int c_lo = split_cols ? eg * (NQ / 2) : 0;
         const int c_hi = split_cols ? c_lo + NQ / 2 : NQ;
         const float invG = 1.f / (float)G;
-        for (int t = split_cols ? 0 : eg; t < ntiles; t += split_cols ? 1 : 2) {
-            const int b = NBUF == 2 ? (t & 1) : 0;
-            const uint32_t bph = NBUF == 2 ? ((t >> 1) & 1) : (t & 1);
-            if (!wait_or_flag(smem_addr(&bar_afull[b]), bph, abort_flag, err)) break;
-            tc_fence_after();
-            const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * 256);
-            float acc = 0.f;
-            for (int cb = c_lo; cb < c_hi; cb += 32) {
-                float v[32];
-                tmem_ld32(ta + cb, v);
+        float *bs = bsh[warp - 4];
+        int gt = 0;
+        long prev_u = -1;
+        for (int i = i_begin; i < i_end; ++i) {
+            const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+            if (it.ntiles == 0) continue;
+            if (it.u != prev_u) {  // this unit's row normalisers (warp-private copy)
+                __syncwarp();
+                for (int rr = lane; rr < kTcMaxR; rr += 32) bs[rr] = rr < R ? rowb[it.u * R + rr] : 0.f;
+                __syncwarp();
+                prev_u = it.u;
+            }
+            bool ok = true;
+            for (int t = 0; t < it.ntiles; ++t, ++gt) {
+                const bool mine = split_cols || ((gt & 1) == eg);
+                if (!mine) continue;
+                const int b = NBUF == 2 ? (gt & 1) : 0;
+                const uint32_t bph = NBUF == 2 ? ((gt >> 1) & 1) : (gt & 1);
+                if (!wait_or_flag(smem_addr(&bar_afull[b]), bph, abort_flag, err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * 256);
+                float acc = 0.f;
+                for (int cb = c_lo; cb < c_hi; cb += 32) {
+                    float v[32];
+                    tmem_ld32(ta + cb, v);
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (cb + i < R) acc += fast_exp2(fmaf(v[i], c2, -bsh[cb + i]));
+                    for (int q = 0; q < 32; ++q)
+                        if (cb + q < R) acc += fast_exp2(fmaf(v[q], c2, -bs[cb + q]));
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
+                const int j = it.j0 + t * 128 + row;
+                if (j < it.j1) {
+                    if (split_cols)  // two halves land on a zeroed entry: 0 + a + b, order-independent
+                        atomicAdd(raw + it.u * L_cap + j, acc * invG);
+                    else
+                        raw[it.u * L_cap + j] = acc * invG;
+                }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
-            const int j = j0 + t * 128 + row;
-            if (j < j1) {
-                if (split_cols)  // two halves land on a zeroed entry: 0 + a + b, order-independent
-                    atomicAdd(raw + u * L_cap + j, acc * invG);
-                else
-                    raw[u * L_cap + j] = acc * invG;
-            }
+            if (!ok) break;
         }
     }
     __syncthreads();
@@ -405,7 +502,6 @@ __global__ void __launch_bounds__(128 + 256, 1)
 }
 
 // ---------------------------------------------------------------- host side
-constexpr int kTcMaxR = 448;  // keeps pass 2 (queries + 3 K stages) within 227 KB of shared memory
 
 int score_tc_nq(int R) { return R <= 256 ? ((R + 15) / 16) * 16 : ((R + 31) / 32) * 32; }
 
@@ -436,8 +532,11 @@ static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t
     cudaError_t e = cudaFuncSetAttribute(score_rowstats_tc<D, N, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    score_rowstats_tc<D, N, MT><<<dim3(nch, (unsigned)units), 128 + 128 * MT, smem, s>>>(
-        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, nch, c2, ws.part_m, ws.part_z, err);
+    const int n_items = (int)(units * nch);
+    const int grid = min(n_items, device_sm_count());
+    score_rowstats_tc<D, N, MT><<<grid, 128 + 128 * MT, smem, s>>>(mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q,
+                                                                  kv.H_kv, kv.L_cap, R, nch, n_items, c2,
+                                                                  ws.part_m, ws.part_z, err);
     *ok = true;
     return cudaGetLastError();
 }
@@ -486,8 +585,10 @@ static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t
     const size_t smem = 1024 + (size_t)(D / 64) * NQ * 128 + 3 * (size_t)(D / 64) * 128 * 128;
     e = cudaFuncSetAttribute(score_colsum_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    score_colsum_tc<D><<<dim3(nch, (unsigned)units), 128 + 256, smem, s>>>(
-        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, NQ, c2, ws.rowb, ws.raw, err);
+    const int n_items = (int)(units * nch);
+    const int grid = min(n_items, device_sm_count());
+    score_colsum_tc<D><<<grid, 128 + 256, smem, s>>>(mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R,
+                                                     NQ, nch, n_items, c2, ws.rowb, ws.raw, err);
     *ok = true;
     return cudaGetLastError();
 }
