@@ -55,6 +55,24 @@ __device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t 
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// 32 consecutive fp32 columns of the calling thread's TMEM lane (no wait: call
+// tmem_ld_wait() before using the values).
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
 // 32 consecutive fp32 columns of the calling thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
 {
@@ -276,27 +294,38 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
                 const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((b * MT + mt) * N);
                 const int jb = it.j0 + t * N;
                 const int lim = min(it.j1 - 1, jmax) - jb;  // columns 0..lim are visible to this row
-#pragma unroll 1
-                for (int cc = 0; cc < N; cc += 32) {
-                    float v[32];
-                    tmem_ld32(ta + cc, v);
-                    float mx = -INFINITY;
+                float v[N];  // the whole tile row: all TMEM loads issued before one wait
 #pragma unroll
-                    for (int q = 0; q < 32; ++q) {
-                        v[q] *= c2;
-                        if (cc + q <= lim) mx = fmaxf(mx, v[q]);
-                    }
-                    const float mn = fmaxf(m, mx);
-                    if (mn == -INFINITY) continue;
-                    float acc = 0.f;
-#pragma unroll
-                    for (int q = 0; q < 32; ++q) acc += (cc + q <= lim) ? fast_exp2(v[q] - mn) : 0.f;
-                    z = z * fast_exp2(m - mn) + acc;
-                    m = mn;
-                }
+                for (int cc = 0; cc < N; cc += 32) tmem_ld32_nowait(ta + cc, *reinterpret_cast<float(*)[32]>(v + cc));
+                tmem_ld_wait();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
+                // logits are v * c2 with c2 > 0: take the max on v, exponentiate fma(v, c2, -m)
+                float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                const bool full_tile = lim >= N - 1;  // no masking needed (most tiles)
+                if (full_tile) {
+#pragma unroll
+                    for (int q = 0; q < N; ++q) mx4[q & 3] = fmaxf(mx4[q & 3], v[q]);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < N; ++q)
+                        if (q <= lim) mx4[q & 3] = fmaxf(mx4[q & 3], v[q]);
+                }
+                const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+                const float mn = fmaxf(m, mx * c2);
+                if (mn == -INFINITY) continue;
+                const float nb = -mn;
+                float a4[4] = {0.f, 0.f, 0.f, 0.f};
+                if (full_tile) {
+#pragma unroll
+                    for (int q = 0; q < N; ++q) a4[q & 3] += fast_exp2(fmaf(v[q], c2, nb));
+                } else {
+#pragma unroll
+                    for (int q = 0; q < N; ++q) a4[q & 3] += (q <= lim) ? fast_exp2(fmaf(v[q], c2, nb)) : 0.f;
+                }
+                z = z * fast_exp2(m - mn) + ((a4[0] + a4[1]) + (a4[2] + a4[3]));
+                m = mn;
             }
             if (!ok) break;
             if (r < R) {
@@ -472,14 +501,25 @@ __global__ void __launch_bounds__(128 + 256, 1)
                 }
                 tc_fence_after();
                 const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * 256);
-                float acc = 0.f;
-                for (int cb = c_lo; cb < c_hi; cb += 32) {
-                    float v[32];
-                    tmem_ld32(ta + cb, v);
+                float a4[4] = {0.f, 0.f, 0.f, 0.f};
+                for (int cb = c_lo; cb < c_hi; cb += 64) {
+                    float v[64];
+                    const bool two = cb + 32 < c_hi;
+                    tmem_ld32_nowait(ta + cb, *reinterpret_cast<float(*)[32]>(v));
+                    if (two) tmem_ld32_nowait(ta + cb + 32, *reinterpret_cast<float(*)[32]>(v + 32));
+                    tmem_ld_wait();
+                    const int nv = two ? 64 : 32;
+                    if (cb + nv <= R) {  // every column is a real window row
 #pragma unroll
-                    for (int q = 0; q < 32; ++q)
-                        if (cb + q < R) acc += fast_exp2(fmaf(v[q], c2, -bs[cb + q]));
+                        for (int q = 0; q < 64; ++q)
+                            if (q < nv) a4[q & 3] += fast_exp2(fmaf(v[q], c2, -bs[cb + q]));
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 64; ++q)
+                            if (q < nv && cb + q < R) a4[q & 3] += fast_exp2(fmaf(v[q], c2, -bs[cb + q]));
+                    }
                 }
+                const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_addr(&bar_aempty[b]));
