@@ -55,7 +55,12 @@ def _load():
     if _lib is not None:
         return _lib
     build()
-    lib = ctypes.CDLL(str(_LIB_PATH))
+    _lib = _bind(ctypes.CDLL(str(_LIB_PATH)))
+    return _lib
+
+
+def _bind(lib):
+    """Declare the C signatures on a loaded oracle library."""
     c_int, c_double, c_float = ctypes.c_int, ctypes.c_double, ctypes.c_float
     lib.oracle_retention_ratio.argtypes = [_f32p, c_int, c_double, c_double]
     lib.oracle_retention_ratio.restype = c_double
@@ -89,7 +94,6 @@ def _load():
     lib.oracle_answer_ppl.argtypes = [_f32p, _i32p, ctypes.c_void_p, c_int, c_int, c_int, c_float,
                                       _f64p, _u8p]
     lib.oracle_answer_ppl.restype = None
-    _lib = lib
     return lib
 
 
