@@ -423,13 +423,59 @@ def run_e2e(hp, wl, args, world):
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n}
 
 
+def run_trace(args):
+    """The step-loop trace (batch 16, 8192 generated tokens, 7B-class heads): one run, timed."""
+    from paper_2608_04771_gb300 import build as B
+    from paper_2608_04771_gb300 import reco, trace
+    B.build()
+    spec = trace.full_trace_spec(args.reading)
+    if args.generated:
+        spec.generated = args.generated
+    warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64)
+    warm.run(max_tokens=128)
+    torch.cuda.synchronize()
+    tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.perf_counter()
+    a.record()
+    ev = tr.run()
+    b.record()
+    b.synchronize()
+    wall = time.perf_counter() - t0
+    reco.reco_check()
+    ms = a.elapsed_time(b)
+    wl = tr.wl
+    row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes
+    full_peak = spec.batch * (spec.prompt + spec.generated) * row_bytes
+    line = {
+        "metric": "step-loop trace: generated tokens/s (decode + penalty every token, compression at step "
+                  "boundaries, answer probes), 1xGB300",
+        "value": ev.generated / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1, "ms_total": ms, "wall_s": wall,
+        "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"trace: 7B-class heads, 28 layers, batch {spec.batch}, prompt {spec.prompt}, "
+                               f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
+                               f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
+                   "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically"},
+        "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
+                  "compressions": ev.compressions, "probes": len(ev.probes),
+                  "stops": sum(1 for p in ev.probes if p[2]),
+                  "peak_cache_bytes": ev.peak_cache_bytes,
+                  "mean_cache_bytes": ev.cache_byte_tokens / max(ev.tokens, 1),
+                  "uncompressed_peak_cache_bytes": full_peak},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
-    ap.add_argument("--workload", default="7b", choices=["tiny", "1.5b", "7b", "32b"])
+    ap.add_argument("--workload", default="7b", choices=["tiny", "1.5b", "7b", "32b", "trace"])
+    ap.add_argument("--reading", default="A", choices=["A", "B"], help="trace: budget base reading")
+    ap.add_argument("--generated", type=int, default=0, help="trace: generated tokens (default 8192)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-units", type=int, default=32, help="oracle sample: units of layer 0")
@@ -439,6 +485,8 @@ def main():
     ap.add_argument("--decode-steps", type=int, help="override the decode steps (profiling a smaller case)")
     args = ap.parse_args()
     from paper_2608_04771_gb300 import workloads as W
+    if args.workload == "trace":
+        return run_trace(args)
     wl = W.WORKLOADS[args.workload]
     over = {k: v for k, v in (("layers", args.layers), ("batch", args.batch),
                                ("decode_steps", args.decode_steps)) if v is not None}

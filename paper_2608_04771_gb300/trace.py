@@ -6,9 +6,11 @@ synthetic).  Per token, every active sequence decodes one token (append + attent
 over its ragged cache, all layers in one call) and the reflection penalty (Eq. 3-4)
 is applied to that token's logits with the band of the sequence's latest reward.
 When a sequence completes a step it receives a reward v_i (Sec. 3.1), and
-  * its cache is compressed to m_i = lambda_i * L (Eq. 1-2, Sec. 3.2) -- all
-    sequences are passed to one scoring/selection call, the others with keep = L,
-    which leaves them untouched;
+  * if its cache has grown by at least S tokens since its last compression
+    (L - L_{i-1} >= S, Sec. 3.2; L_0 = the prompt; S = 0 compresses at every
+    step boundary) it is compressed to m_i = lambda_i * L (Eq. 1-2, Sec. 3.2) --
+    all sequences are passed to one scoring/selection call, the others with
+    keep = L, which leaves them untouched;
   * if v_{i-1} >= tau_h and v_i >= tau_h, the answer probe runs (Eq. 5-6) and a
     sequence that passes PPL <= tau_p stops and leaves the batch.
 Budget base L (the paper is silent on repeated compression): reading "A" uses the
@@ -38,6 +40,7 @@ class TraceSpec:
     seed: int
     reading: str = "A"
     L_cap: int = 0  # rows per unit; 0 = choose from the reading
+    interval: int = 0  # S: minimum growth since the last compression (0: every step boundary)
 
     def cap(self) -> int:
         if self.L_cap:
@@ -55,13 +58,21 @@ def full_trace_spec(reading="A") -> TraceSpec:
 class TraceEvents:
     """What the loop did, for replay and checks."""
     boundaries: list = field(default_factory=list)  # (token, [(seq, reward, keep)], stops)
-    probes: list = field(default_factory=list)      # (token, seq, stopped)
-    tokens: int = 0
+    probes: list = field(default_factory=list)      # (token, seq, stopped, ppl)
+    tokens: int = 0            # decode launches (loop iterations)
+    generated: int = 0         # tokens generated, summed over sequences
+    steps_completed: int = 0   # step boundaries, summed over sequences
+    compressions: int = 0      # per-sequence compressions
+    peak_cache_bytes: int = 0  # max over tokens of the K+V bytes held by the active sequences
+    cache_byte_tokens: float = 0.0  # sum over tokens of the K+V bytes held (for the mean)
 
 
 class Trace:
-    def __init__(self, spec: TraceSpec, device="cuda", out_dtype=torch.float32):
+    def __init__(self, spec: TraceSpec, device="cuda", out_dtype=torch.float32, input_pool: int = 0):
+        """input_pool > 0: per-token inputs are drawn once for that many tokens and reused
+        cyclically (timing runs); 0: every token draws its own seeded inputs."""
         self.spec = spec
+        self.input_pool = input_pool
         wl = spec.base.reduced(batch=spec.batch, L=spec.prompt, decode_steps=spec.cap() - spec.prompt,
                                seed=spec.seed)
         self.wl = wl
@@ -75,22 +86,36 @@ class Trace:
         self.lens = [spec.prompt] * spec.batch  # per active sequence (all its units share it)
         self.full = [spec.prompt] * spec.batch  # uncompressed length so far
         self.hist = [[] for _ in range(spec.batch)]
+        self.last_comp = [spec.prompt] * spec.batch  # L_{i-1}: length after the last compression
         self.step_idx = [0] * spec.batch
         self.out_dtype = out_dtype
         self.ids = torch.from_numpy(W.make_reflection_ids(wl)).to(device) if wl.vocab else None
+        self._pool = None
+        if input_pool:
+            self._pool = [(self._token_inputs(t), self._window_queries(t) if t < 8 else None,
+                           self._token_logits(t) if wl.vocab else None) for t in range(input_pool)]
         self._rebuild()
 
     # ---------------------------------------------------------------- inputs
-    def token_inputs(self, t: int):
-        """q [Ly, B, Hq, d], k_new / v_new [Ly, B, Hkv, d] for token t, full batch."""
+    def _token_inputs(self, t: int):
         return W.make_decode_step(self.wl, 1000 + t, self.device)
 
-    def window_queries(self, t: int):
+    def _window_queries(self, t: int):
         wl = self.wl
         return W.randn((wl.layers, wl.batch, wl.h_q, wl.w, wl.d), wl, 5_000_000 + t, self.device)
 
-    def token_logits(self, t: int):
+    def _token_logits(self, t: int):
         return W.randn((self.wl.batch, self.wl.vocab), self.wl, 9_000_000 + t, self.device, torch.float32) * 2.0
+
+    def token_inputs(self, t: int):
+        """q [Ly, B, Hq, d], k_new / v_new [Ly, B, Hkv, d] for token t, full batch."""
+        return self._pool[t % self.input_pool][0] if self._pool else self._token_inputs(t)
+
+    def window_queries(self, t: int):
+        return self._pool[t % 8][1] if self._pool else self._window_queries(t)
+
+    def token_logits(self, t: int):
+        return self._pool[t % self.input_pool][2].clone() if self._pool else self._token_logits(t)
 
     def answer(self, t: int, seq: int):
         """Answer logits / tokens of a probe of sequence `seq` at token t (confident on even probes)."""
@@ -122,6 +147,7 @@ class Trace:
         self.active = [self.active[i] for i in keep_pos]
         self.lens = [self.lens[i] for i in keep_pos]
         self.full = [self.full[i] for i in keep_pos]
+        self.last_comp = [self.last_comp[i] for i in keep_pos]
         self._rebuild()
 
     def current_reward(self, s: int) -> float:
@@ -143,6 +169,11 @@ class Trace:
             reco.reco_decode_attn(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, lse, self.ws_decode)
             self.lens = [L + 1 for L in self.lens]
             self.full = [F + 1 for F in self.full]
+            ev.generated += len(self.active)
+            row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes  # K and V of one token
+            held = sum(self.lens) * row_bytes
+            ev.peak_cache_bytes = max(ev.peak_cache_bytes, held)
+            ev.cache_byte_tokens += held
             logits = None
             if self.ids is not None:
                 logits = self.token_logits(t).index_select(0, torch.tensor(self.active, device=self.device))
@@ -162,21 +193,28 @@ class Trace:
                     done.append(i)
             if not done:
                 continue
+            ev.steps_completed += len(done)
             keep = list(self.lens)
             info = []
             for i in done:
                 s = self.active[i]
+                if self.lens[i] - self.last_comp[i] < spec.interval:
+                    continue  # grown by less than S since the last compression
                 ratio = reco.reco_retention_ratio(np.array(self.hist[s], np.float32), wl.base, wl.delta)
                 base_len = self.lens[i] if spec.reading == "A" else self.full[i]
                 m = reco.reco_keep_count(ratio, base_len, wl.w)
                 keep[i] = min(m, self.lens[i])
+                self.last_comp[i] = keep[i]
                 info.append((s, float(self.hist[s][-1]), keep[i]))
-            q_win = sel(self.window_queries(t))
-            keep_dev = torch.tensor(keep, dtype=torch.int32, device=self.device)
-            reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
-                                  self.ws_score)
-            reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
-                                     self.ws_select)
+                ev.compressions += 1
+            q_win = None
+            if info:
+                q_win = sel(self.window_queries(t))
+                keep_dev = torch.tensor(keep, dtype=torch.int32, device=self.device)
+                reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
+                                      self.ws_score)
+                reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
+                                         self.ws_select)
             if on_boundary:
                 on_boundary(t, self, done, keep, q_win)
             self.lens = keep

@@ -38,6 +38,7 @@ class OracleReplay:
         self.K = np32(tr.K).astype(np.float32)  # [Ly, B, Hkv, L_cap, d], original batch order
         self.V = np32(tr.V).astype(np.float32)
         self.lens = {s: tr.spec.prompt for s in range(tr.spec.batch)}
+        self.last_comp = {s: tr.spec.prompt for s in range(tr.spec.batch)}
         self.hist = {s: [] for s in range(tr.spec.batch)}
         self.ids = W.make_reflection_ids(wl)
         self.checked_tokens = 0
@@ -79,7 +80,7 @@ class OracleReplay:
     def on_boundary(self, t, tr, done, keep, q_win):
         wl = self.wl
         act = list(tr.active)
-        qw = np32(q_win)
+        qw = np32(q_win) if q_win is not None else None
         got_kept = tr.kept.cpu().numpy()
         got_scores = tr.scores.cpu().numpy()
         for i in done:
@@ -90,8 +91,11 @@ class OracleReplay:
             hs = self.hist[s]
             if len(hs) >= 2 and oracle.probe_trigger(hs[-2], hs[-1], wl.tau_h):
                 self.expected_probes.add((t, s))
-            ratio = oracle.retention_ratio(np.array(hs, np.float32), wl.base, wl.delta)
             L = self.lens[s]
+            if L - self.last_comp[s] < tr.spec.interval:  # grown by less than S: no compression
+                assert keep[i] == L
+                continue
+            ratio = oracle.retention_ratio(np.array(hs, np.float32), wl.base, wl.delta)
             base_len = L if tr.spec.reading == "A" else tr.spec.prompt + t + 1
             m = min(oracle.keep_count(ratio, base_len, wl.w), L)
             assert m == keep[i], (t, s, m, keep[i])
@@ -110,6 +114,7 @@ class OracleReplay:
                     self.K[l, s, h, :m] = oracle.gather_unit(self.K[l, s, h, :L], idx)
                     self.V[l, s, h, :m] = oracle.gather_unit(self.V[l, s, h, :L], idx)
             self.lens[s] = m
+            self.last_comp[s] = m
         self.checked_boundaries += 1
 
 
@@ -137,6 +142,17 @@ def test_trace_reading_A_reduced():
     assert rep.tie_diffs == 0  # no near-tie flips on this seed: every unit compared throughout
     assert rep.checked_tokens >= 150 and rep.checked_boundaries >= 15
     assert len(ev.probes) == 4 and sum(st for (_, _, st, _) in ev.probes) == 3
+
+
+def test_trace_interval_trigger():
+    """Compress only once the cache has grown by S = 100 tokens since the last compression."""
+    base = W.WORKLOADS["7b"].reduced(layers=1, vocab=2000)
+    spec = trace.TraceSpec(base, batch=3, prompt=64, generated=420, step_mean=30, step_min=8, seed=7,
+                           reading="A", interval=100)
+    tr, rep, ev = _run(spec)
+    assert rep.tie_diffs == 0
+    assert 0 < ev.compressions < ev.steps_completed  # some boundaries skip compression
+    assert ev.peak_cache_bytes > 0 and ev.generated > 0
 
 
 def test_trace_reading_B_reduced_with_stops():
