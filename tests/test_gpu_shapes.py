@@ -1,0 +1,48 @@
+"""Head shapes, windows, pool widths and dtypes beyond the named workloads, each run
+score -> select/compact -> decode against the oracle (see test_gpu_pipeline)."""
+import ctypes
+
+import pytest
+import torch
+
+from paper_2608_04771_gb300 import reco
+from paper_2608_04771_gb300 import workloads as W
+from test_gpu_pipeline import run_pipeline
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2608_04771_gb300 import build
+    build.build()
+    reco.lib()
+
+
+BASE = W.WORKLOADS["7b"]
+CASES = {
+    # name: overrides                                       path exercised
+    "mha_g1": dict(h_q=4, h_kv=4, w=16, L=900),            # G = 1
+    "g3_d64_pool3": dict(h_q=6, h_kv=2, w=8, d=64, pool=3, L=700),
+    "g8_r256": dict(h_q=16, h_kv=2, w=32, L=1300),         # tensor decode at G = 8; pass 2 N = 256
+    "g16_simt_decode": dict(h_q=16, h_kv=1, w=16, L=800),  # G = 16: bf16 decode on the SIMT path
+    "w1_pool1": dict(w=1, pool=1, L=600),                  # one window query, Eq. 2 without pooling
+    "r320_pool9": dict(h_q=10, h_kv=2, w=64, pool=9, L=1500),  # split-column pass 2
+    "r384_max": dict(h_q=12, h_kv=2, w=64, L=1000),        # largest tensor-core window
+    "fp32_d128": dict(dtype="f32", d=128, L=600),
+}
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_pipeline_shape(name):
+    wl = BASE.reduced(layers=1, batch=2, decode_steps=2, **CASES[name])
+    run_pipeline(wl)
+
+
+def test_window_rows_beyond_both_scoring_paths_are_rejected():
+    wl = BASE.reduced(layers=1, batch=1, h_q=8, h_kv=1, w=64, L=300, decode_steps=0)  # G*w = 512
+    K, V = W.make_cache(wl, "cuda", canary=False)
+    kv = reco.make_kv(K, V, wl.h_q)
+    st = reco.lib().reco_score_cache(ctypes.byref(kv), ctypes.c_void_p(K.data_ptr()), ctypes.c_void_p(16),
+                                     wl.w, 7, 0.1, ctypes.c_void_p(16), ctypes.c_void_p(256 * 4096), 1 << 40, None)
+    assert st == reco.RECO_EUNSUPPORTED
