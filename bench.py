@@ -431,10 +431,11 @@ def run_trace(args):
     spec = trace.full_trace_spec(args.reading)
     if args.generated:
         spec.generated = args.generated
-    warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64)
+    use_graph = not args.no_graph
+    warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64, use_graph=use_graph)
     warm.run(max_tokens=128)
     torch.cuda.synchronize()
-    tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64)
+    tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64, use_graph=use_graph)
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.perf_counter()
@@ -456,7 +457,9 @@ def run_trace(args):
         "config": {"workload": f"trace: 7B-class heads, 28 layers, batch {spec.batch}, prompt {spec.prompt}, "
                                f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
                                f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
-                   "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically"},
+                   "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically",
+                   "per_token_launch": "captured CUDA graph (decode + penalty)" if use_graph
+                   else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),
                   "stops": sum(1 for p in ev.probes if p[2]),
@@ -476,6 +479,7 @@ def main():
     ap.add_argument("--workload", default="7b", choices=["tiny", "1.5b", "7b", "32b", "trace"])
     ap.add_argument("--reading", default="A", choices=["A", "B"], help="trace: budget base reading")
     ap.add_argument("--generated", type=int, default=0, help="trace: generated tokens (default 8192)")
+    ap.add_argument("--no-graph", action="store_true", help="trace: per-token calls without a CUDA graph")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-units", type=int, default=32, help="oracle sample: units of layer 0")

@@ -17,6 +17,10 @@ Budget base L (the paper is silent on repeated compression): reading "A" uses th
 current cache length, reading "B" the full uncompressed length so far (the keep
 count is then capped at the current length).  Lengths are tracked on the host, so
 the loop needs no device read-back except the stop flags of a probe.
+
+With use_graph, a token's decode + penalty is one captured CUDA graph over static
+input buffers (captured again whenever the batch shrinks), so the per-token host
+work is one input copy and one graph launch.
 """
 from __future__ import annotations
 
@@ -27,6 +31,29 @@ import torch
 
 from . import reco
 from . import workloads as W
+
+
+def _pack(parts, out=None):
+    """Lay tensors end to end in one uint8 buffer (each part 256-byte aligned); returns the
+    buffer and a view of each part in it.  With `out`, views into `out` are made instead
+    (the parts then only give shapes and dtypes)."""
+    offs, n = [], 0
+    for x in parts:
+        offs.append(n)
+        n += (x.numel() * x.element_size() + 255) // 256 * 256
+    buf = out if out is not None else torch.empty(n, dtype=torch.uint8, device=parts[0].device)
+    views = []
+    for x, o in zip(parts, offs):
+        v = buf[o:o + x.numel() * x.element_size()].view(x.dtype).view(x.shape)
+        if out is None:
+            v.copy_(x)
+        views.append(v)
+    return buf, views
+
+
+def _to_device(values, dtype, device):
+    """Host list -> device tensor through pinned memory, without blocking the host."""
+    return torch.tensor(values, dtype=dtype).pin_memory().to(device, non_blocking=True)
 
 
 @dataclass
@@ -68,19 +95,28 @@ class TraceEvents:
 
 
 class Trace:
-    def __init__(self, spec: TraceSpec, device="cuda", out_dtype=torch.float32, input_pool: int = 0):
+    def __init__(self, spec: TraceSpec, device="cuda", out_dtype=torch.float32, input_pool: int = 0,
+                 use_graph: bool = False):
         """input_pool > 0: per-token inputs are drawn once for that many tokens and reused
-        cyclically (timing runs); 0: every token draws its own seeded inputs."""
+        cyclically (timing runs); 0: every token draws its own seeded inputs.
+        use_graph: the per-token decode + penalty runs as a captured CUDA graph."""
         self.spec = spec
         self.input_pool = input_pool
+        self.use_graph = use_graph
+        self.graph = None
         wl = spec.base.reduced(batch=spec.batch, L=spec.prompt, decode_steps=spec.cap() - spec.prompt,
                                seed=spec.seed)
         self.wl = wl
         self.device = device
         self.steps = W.make_trace_steps(spec.batch, spec.generated, spec.step_mean, spec.step_min, spec.seed)
         self.rewards = W.make_trace_rewards(self.steps, spec.seed)
-        # token index at which each step of each sequence completes
+        # token index at which each step of each sequence completes, and its inverse
+        # (token -> the sequences that complete a step there)
         self.ends = [np.cumsum(s) - 1 for s in self.steps]
+        self.ends_at = {}
+        for sq, e in enumerate(self.ends):
+            for tok in e.tolist():
+                self.ends_at.setdefault(tok, []).append(sq)
         self.K, self.V = W.make_cache(wl, device, canary=False)
         self.active = list(range(spec.batch))  # original sequence ids, in batch order
         self.lens = [spec.prompt] * spec.batch  # per active sequence (all its units share it)
@@ -125,10 +161,47 @@ class Trace:
             z = W.randn(z.shape, wl, 12, self.device, torch.float32) * 2.0
         return z, tok
 
+    def _full_batch(self) -> bool:
+        return len(self.active) == self.spec.batch
+
+    def _sel(self, x, dim=1):
+        """Rows of the active sequences (batch dimension `dim`), in batch order."""
+        return x if self._full_batch() else x.index_select(dim, self.idx_dev).contiguous()
+
+    def active_inputs(self, t: int):
+        """Token t's q, k_new, v_new for the active sequences."""
+        if self._apool is not None:
+            return self._apool[t % self.input_pool][1]
+        q, kn, vn = self._token_inputs(t)
+        return self._sel(q), self._sel(kn), self._sel(vn)
+
+    def active_logits(self, t: int):
+        """A fresh copy of token t's logits rows of the active sequences."""
+        if self._apool is not None:
+            return self._apool[t % self.input_pool][2].clone()
+        return self._sel(self._token_logits(t), 0)
+
     # ---------------------------------------------------------------- plumbing
+    def _active_pool(self):
+        """The input pool restricted to the active sequences.  Each slot's q | k_new | v_new
+        | logits are packed into one byte buffer laid out like the captured graph's static
+        inputs, so a token's inputs arrive in a single copy."""
+        if not self._pool:
+            return None
+        apool = []
+        for (q, kn, vn), _, z in self._pool:
+            parts = [self._sel(q), self._sel(kn), self._sel(vn)] + ([] if z is None else [self._sel(z, 0)])
+            packed, views = _pack(parts)
+            apool.append((packed, tuple(views[:3]), views[3] if z is not None else None))
+        return apool
+
     def _rebuild(self):
         wl = self.wl
         self.B = len(self.active)
+        self.pos = {sq: i for i, sq in enumerate(self.active)}  # sequence id -> batch position
+        self.idx_dev = torch.tensor(self.active, dtype=torch.long, device=self.device)
+        self._apool = None
+        self._apool = self._active_pool()
         self.kv = reco.make_kv(self.K, self.V, wl.h_q)
         self.ws_score = reco.workspace(reco.RECO_OP_SCORE, self.kv, wl.w, self.device)
         self.ws_select = reco.workspace(reco.RECO_OP_SELECT, self.kv, wl.w, self.device)
@@ -138,6 +211,7 @@ class Trace:
         self.lens_dev = torch.tensor(self.lens, dtype=torch.int32, device=self.device).view(1, -1, 1).expand(
             wl.layers, -1, wl.h_kv).contiguous()
         self.ws_ppl = reco.workspace(reco.RECO_OP_PPL, None, wl.n_answer, self.device)
+        self.graph = None  # buffers and pointers changed: capture again before the next token
 
     def _drop(self, gone):
         keep_pos = [i for i, s in enumerate(self.active) if s not in gone]
@@ -150,49 +224,95 @@ class Trace:
         self.last_comp = [self.last_comp[i] for i in keep_pos]
         self._rebuild()
 
+    def _capture(self):
+        """Static input/output buffers and one CUDA graph of a token's decode + penalty."""
+        wl, dev, B = self.wl, self.device, len(self.active)
+        shapes = [((wl.layers, B, wl.h_q, wl.d), wl.torch_dtype), ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype),
+                  ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype)]
+        if self.ids is not None:
+            shapes.append(((B, wl.vocab), torch.float32))
+        protos = [torch.empty(sh, dtype=dt, device="meta") for sh, dt in shapes]
+        n = sum((x.numel() * x.element_size() + 255) // 256 * 256 for x in protos)
+        self.g_in = torch.zeros(n, dtype=torch.uint8, device=dev)  # q | k_new | v_new | logits
+        _, views = _pack(protos, out=self.g_in)
+        self.g_q, self.g_kn, self.g_vn = views[:3]
+        self.g_logits = views[3] if self.ids is not None else None
+        self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
+        self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
+        self.g_rw = _to_device([self.current_reward(s) for s in self.active], torch.float32, dev)
+        # one call outside the capture, without an append (cache and lens stay as they are)
+        reco.reco_decode_attn(self.kv, self.g_q, None, None, self.lens_dev, wl.scale(), self.g_out, self.g_lse,
+                              self.ws_decode)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="relaxed"):
+            reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
+                                  self.g_lse, self.ws_decode)
+            if self.g_logits is not None:
+                reco.reco_reflect_penalty(self.g_logits, self.ids, self.g_rw, wl.tau_l, wl.tau_h, wl.beta)
+        self.graph = g
+
     def current_reward(self, s: int) -> float:
         return float(self.hist[s][-1]) if self.hist[s] else 0.0
 
     # ---------------------------------------------------------------- the loop
+    def _token(self, t: int):
+        """Decode (append + attention) and penalty of token t; returns out, lse, logits."""
+        wl = self.wl
+        if self.use_graph:
+            if self.graph is None:
+                self._capture()
+            if self._apool is not None:
+                self.g_in.copy_(self._apool[t % self.input_pool][0])
+            else:
+                q, kn, vn = self.active_inputs(t)
+                self.g_q.copy_(q)
+                self.g_kn.copy_(kn)
+                self.g_vn.copy_(vn)
+                if self.g_logits is not None:
+                    self.g_logits.copy_(self.active_logits(t))
+            self.graph.replay()
+            return self.g_out, self.g_lse, self.g_logits
+        q, kn, vn = self.active_inputs(t)
+        out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=self.device)
+        reco.reco_decode_attn(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, lse, self.ws_decode)
+        logits = None
+        if self.ids is not None:
+            logits = self.active_logits(t)
+            rw = _to_device([self.current_reward(s) for s in self.active], torch.float32, self.device)
+            reco.reco_reflect_penalty(logits, self.ids, rw, wl.tau_l, wl.tau_h, wl.beta)
+        return out, lse, logits
+
     def run(self, max_tokens=None, on_token=None, on_boundary=None) -> TraceEvents:
         spec, wl = self.spec, self.wl
         ev = TraceEvents()
         T = spec.generated if max_tokens is None else min(max_tokens, spec.generated)
-        sel = lambda x: x.index_select(1, torch.tensor(self.active, device=self.device)).contiguous()  # noqa: E731
+        row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes  # K and V of one token
         for t in range(T):
             if not self.active:
                 break
-            q, kn, vn = self.token_inputs(t)
-            q, kn, vn = sel(q), sel(kn), sel(vn)
-            out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
-            lse = torch.empty(q.shape[:3], dtype=torch.float32, device=self.device)
-            reco.reco_decode_attn(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, lse, self.ws_decode)
+            out, lse, logits = self._token(t)
             self.lens = [L + 1 for L in self.lens]
             self.full = [F + 1 for F in self.full]
             ev.generated += len(self.active)
-            row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes  # K and V of one token
             held = sum(self.lens) * row_bytes
             ev.peak_cache_bytes = max(ev.peak_cache_bytes, held)
             ev.cache_byte_tokens += held
-            logits = None
-            if self.ids is not None:
-                logits = self.token_logits(t).index_select(0, torch.tensor(self.active, device=self.device))
-                rw = torch.tensor([self.current_reward(s) for s in self.active], dtype=torch.float32,
-                                  device=self.device)
-                reco.reco_reflect_penalty(logits, self.ids, rw, wl.tau_l, wl.tau_h, wl.beta)
             if on_token:
                 on_token(t, self, out, lse, logits)
             ev.tokens += 1
-            # step boundaries completed at this token
+            # step boundaries completed at this token (batch positions, in batch order)
             done = []
-            for i, s in enumerate(self.active):
-                k = self.step_idx[s]
-                if k < len(self.ends[s]) and self.ends[s][k] == t:
-                    self.step_idx[s] += 1
-                    self.hist[s].append(self.rewards[s][k])
-                    done.append(i)
+            for s in self.ends_at.get(t, ()):
+                if s not in self.pos:
+                    continue  # stopped earlier
+                self.hist[s].append(self.rewards[s][self.step_idx[s]])
+                self.step_idx[s] += 1
+                done.append(self.pos[s])
             if not done:
                 continue
+            done.sort()
             ev.steps_completed += len(done)
             keep = list(self.lens)
             info = []
@@ -209,8 +329,8 @@ class Trace:
                 ev.compressions += 1
             q_win = None
             if info:
-                q_win = sel(self.window_queries(t))
-                keep_dev = torch.tensor(keep, dtype=torch.int32, device=self.device)
+                q_win = self._sel(self.window_queries(t))
+                keep_dev = _to_device(keep, torch.int32, self.device)
                 reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
                                       self.ws_score)
                 reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
@@ -235,4 +355,7 @@ class Trace:
             ev.boundaries.append((t, info, sorted(gone)))
             if gone:
                 self._drop(gone)
+            elif self.use_graph and self.graph is not None:
+                self.g_rw.copy_(_to_device([self.current_reward(s) for s in self.active], torch.float32,
+                                           self.device))
         return ev

@@ -118,8 +118,8 @@ class OracleReplay:
         self.checked_boundaries += 1
 
 
-def _run(spec, track=None, decode_every=1):
-    tr = trace.Trace(spec, DEV)
+def _run(spec, track=None, decode_every=1, use_graph=False):
+    tr = trace.Trace(spec, DEV, use_graph=use_graph)
     rep = OracleReplay(tr, track, decode_every)
     ev = tr.run(on_token=rep.on_token, on_boundary=rep.on_boundary)
     reco.reco_check()
@@ -133,12 +133,13 @@ def _run(spec, track=None, decode_every=1):
     return tr, rep, ev
 
 
-def test_trace_reading_A_reduced():
+@pytest.mark.parametrize("use_graph", [False, True])
+def test_trace_reading_A_reduced(use_graph):
     # tau_h 0.6 so that this seed's Beta(2,2) rewards trigger probes (4 probes, 3 stops)
     base = W.WORKLOADS["7b"].reduced(layers=2, vocab=5000, tau_h=0.6)
     spec = trace.TraceSpec(base, batch=4, prompt=128, generated=400, step_mean=40, step_min=8, seed=4,
                            reading="A")
-    tr, rep, ev = _run(spec)
+    tr, rep, ev = _run(spec, use_graph=use_graph)
     assert rep.tie_diffs == 0  # no near-tie flips on this seed: every unit compared throughout
     assert rep.checked_tokens >= 150 and rep.checked_boundaries >= 15
     assert len(ev.probes) == 4 and sum(st for (_, _, st, _) in ev.probes) == 3
@@ -170,7 +171,7 @@ def test_trace_full_size_sampled():
     generated tokens, steps of Poisson(96)+16, Beta(2,2) rewards, reading A) with the
     oracle following two whole sequences (decode checked every 8th token, every boundary)."""
     spec = trace.full_trace_spec("A")
-    tr, rep, ev = _run(spec, track=[0, 9], decode_every=8)
+    tr, rep, ev = _run(spec, track=[0, 9], decode_every=8, use_graph=True)
     assert rep.checked_boundaries >= 100 and rep.checked_tokens >= 100
     # near-tie flips (fp32 vs fp64 scores within 1e-5 of the cut) stop the comparison of that unit only
     assert len(rep.diverged) <= 0.05 * 2 * spec.base.layers * spec.base.h_kv, rep.diverged
