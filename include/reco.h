@@ -97,7 +97,7 @@ reco_status reco_check(cudaStream_t stream);
 
 /* ---------------------------------------------------------------- device calls */
 
-/* Eq. 2 (Sec. 3.2, attention-guided selection) for every unit of the cache.
+/* Eq. 2 (Sec. 3.2, attention-guided selection) for the units of the cache.
  * For unit (layer, b, h) of length L = lens[unit] and window w:
  *   logit[g,t,j] = scale * q_win[layer,b,h*G+g,t,:] . K[unit, j, :]
  *   window query t sits at position L-w+t and sees keys j <= L-w+t (causal);
@@ -106,12 +106,18 @@ reco_status reco_check(cudaStream_t stream);
  * for the candidates j in [0, L-w); entries j >= L-w are left unchanged.
  *   q_win  : [n_layers][B][H_q][w][d], same dtype as the cache (device)
  *   lens   : [n_layers][B][H_kv] int32 (device), w <= lens <= L_cap
+ *   keep   : [B] int32 (device) or NULL.  NULL scores every unit.  Given (the keep
+ *            counts the following reco_select_compact call receives), a unit with
+ *            keep[b] >= L is skipped: a sequence that is not compressed this time
+ *            (keep == L, the selection's no-op) costs no key reads, and its rows of
+ *            scores are left unchanged.  Sequences reach step boundaries at
+ *            different tokens (Sec. 3.1), so most calls compress few of them.
  *   scores : [n_layers][B][H_kv][L_cap] float32 (device, written)
  *   pool_kernel: odd, >= 1 (1 = Eq. 2 as printed); scale: e.g. 1/sqrt(d)
  *   ws     : workspace of reco_workspace_bytes(RECO_OP_SCORE, kv, w) bytes
  * A unit with lens outside [w, L_cap] is skipped (device error word set).     */
-reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, int w,
-                             int pool_kernel, float scale, float *scores, void *ws, size_t ws_bytes,
+reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, const int32_t *keep,
+                             int w, int pool_kernel, float scale, float *scores, void *ws, size_t ws_bytes,
                              cudaStream_t stream);
 
 /* Top-m selection and in-place compaction (Sec. 3.2: keep the m_i best tokens,

@@ -224,14 +224,15 @@ reco_status reco_check(cudaStream_t stream)
     return RECO_OK;
 }
 
-reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, int w, int pool_kernel,
-                             float scale, float *scores, void *ws, size_t ws_bytes, cudaStream_t stream)
+reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
+                             int pool_kernel, float scale, float *scores, void *ws, size_t ws_bytes,
+                             cudaStream_t stream)
 {
     reco_status st = check_kv(kv);
     if (st != RECO_OK) return st;
     if (!q_win || !lens || !scores) return fail(RECO_EINVAL, "NULL q_win, lens or scores");
-    if (!al16(q_win) || ((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u))
-        return fail(RECO_EINVAL, "q_win must be 16-byte aligned, lens and scores 4-byte aligned");
+    if (!al16(q_win) || ((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u) || ((uintptr_t)keep & 3u))
+        return fail(RECO_EINVAL, "q_win must be 16-byte aligned, lens, keep and scores 4-byte aligned");
     if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
     if (pool_kernel < 1 || (pool_kernel & 1) == 0) return fail(RECO_EINVAL, "pool_kernel %d must be odd and >= 1", pool_kernel);
     if (!(scale == scale)) return fail(RECO_EINVAL, "scale is NaN");
@@ -243,7 +244,7 @@ reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t
     if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
     unsigned *err;
     if ((st = error_word(&err)) != RECO_OK) return st;
-    cudaError_t e = reco::launch_score(*kv, q_win, lens, w, pool_kernel, scale, scores, lay, err, stream);
+    cudaError_t e = reco::launch_score(*kv, q_win, lens, keep, w, pool_kernel, scale, scores, lay, err, stream);
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_score_cache launch");
 }
 

@@ -15,11 +15,29 @@ constexpr int kDecodeMaxTarget = 16384;
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-struct ScoreWs {  // float regions carved from the caller's workspace
+struct ScoreWs {  // regions carved from the caller's workspace
     float *part_m, *part_z;  // [units][n_chunks][R]  per-chunk row max (log2) / row sum
     float *rowb;             // [units][R]            log2 of the row normaliser
     float *raw;              // [units][L_cap]        unpooled scores
+    int32_t *ulist;          // [units]               units to score, ascending (with a keep mask)
+    int32_t *ucount;         // [1]                   entries of ulist
     size_t bytes;
+};
+
+// Which units a scoring call covers.  With keep == nullptr every unit; otherwise a
+// unit whose sequence keeps its whole cache this time (keep[b] >= lens[unit], the
+// selection's no-op) is skipped: none of its keys are read and its scores are not
+// written.  A unit with an out-of-range length is never skipped, so it still raises
+// the length error.
+struct ScoreMask {
+    const int32_t *keep;  // [B] or nullptr
+    int B, Hkv;
+#ifdef __CUDACC__
+    __device__ __forceinline__ bool skip(long u, int L, int w, int L_cap) const
+    {
+        return keep != nullptr && L >= w && L <= L_cap && keep[(u / Hkv) % B] >= L;
+    }
+#endif
 };
 
 struct SelectWs {
@@ -41,8 +59,8 @@ SelectWs select_ws_layout(const reco_kv &kv, void *base);
 DecodeWs decode_ws_layout(const reco_kv &kv, void *base);
 
 // Launchers return cudaSuccess or the launch error.  All arguments validated by the caller.
-cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, int pool,
-                         float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s);
+cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
+                         int pool, float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s);
 cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
                                   const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
                                   unsigned *err, cudaStream_t s);

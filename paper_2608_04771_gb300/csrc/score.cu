@@ -34,6 +34,8 @@ ScoreWs score_ws_layout(const reco_kv &kv, int w, void *base)
     ws.part_z = (float *)take(units * nch * R * 4);
     ws.rowb = (float *)take(units * R * 4);
     ws.raw = (float *)take(units * (size_t)kv.L_cap * 4);
+    ws.ulist = (int32_t *)take(units * 4);
+    ws.ucount = (int32_t *)take(4);
     ws.bytes = off;
     return ws;
 }
@@ -42,8 +44,8 @@ ScoreWs score_ws_layout(const reco_kv &kv, int w, void *base)
 // through shared memory 64 rows at a time.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) score_rowstats_simt(
-    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, int w,
-    int G, int Hq, int Hkv, int L_cap, int R, int n_chunks, float c2, float *__restrict__ part_m,
+    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, ScoreMask mask,
+    int w, int G, int Hq, int Hkv, int L_cap, int R, int n_chunks, float c2, float *__restrict__ part_m,
     float *__restrict__ part_z, unsigned *err)
 {
     constexpr int KT = 64;
@@ -56,6 +58,7 @@ __global__ void __launch_bounds__(256) score_rowstats_simt(
         if (chunk == 0 && blockIdx.z == 0 && threadIdx.x == 0) raise_error(err, ERR_LEN);
         return;
     }
+    if (mask.skip(u, L, w, L_cap)) return;
     const int j0 = chunk * kScoreChunk;
     const int j1 = min(j0 + kScoreChunk, L);
     const long lb = u / Hkv;
@@ -109,8 +112,8 @@ __global__ void __launch_bounds__(256) score_rowstats_simt(
 }
 
 // Merge the chunk partials of each row into b_r = m_r + log2(Z_r).
-__global__ void score_combine(const int32_t *__restrict__ lens, int w, int L_cap, int R, int n_chunks,
-                              const float *__restrict__ part_m, const float *__restrict__ part_z,
+__global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap, int R,
+                              int n_chunks, const float *__restrict__ part_m, const float *__restrict__ part_z,
                               float *__restrict__ rowb, long units)
 {
     long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -118,7 +121,7 @@ __global__ void score_combine(const int32_t *__restrict__ lens, int w, int L_cap
     long u = i / R;
     int r = (int)(i % R);
     int L = lens[u];
-    if (L < w || L > L_cap) return;
+    if (L < w || L > L_cap || mask.skip(u, L, w, L_cap)) return;
     int used = (L + kScoreChunk - 1) / kScoreChunk;
     float m = -INFINITY, z = 0.f;
     for (int c = 0; c < used; ++c) {
@@ -132,8 +135,8 @@ __global__ void score_combine(const int32_t *__restrict__ lens, int w, int L_cap
 // queries sit in shared memory and are read by broadcast.
 template <typename T, int D>
 __global__ void __launch_bounds__(128) score_colsum_simt(
-    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, int w,
-    int G, int Hq, int Hkv, int L_cap, int R, float c2, const float *__restrict__ rowb,
+    const T *__restrict__ q_win, const T *__restrict__ K, const int32_t *__restrict__ lens, ScoreMask mask,
+    int w, int G, int Hq, int Hkv, int L_cap, int R, float c2, const float *__restrict__ rowb,
     float *__restrict__ raw)
 {
     extern __shared__ __align__(16) float smem[];
@@ -142,7 +145,7 @@ __global__ void __launch_bounds__(128) score_colsum_simt(
     const int chunk = blockIdx.x;
     const long u = blockIdx.y;
     const int L = lens[u];
-    if (L < w || L > L_cap) return;
+    if (L < w || L > L_cap || mask.skip(u, L, w, L_cap)) return;
     const int nc = L - w;
     const int j0 = chunk * kScoreChunk;
     const int j1 = min(j0 + kScoreChunk, nc);
@@ -181,13 +184,13 @@ __global__ void __launch_bounds__(128) score_colsum_simt(
 }
 
 // Max-pool over the clipped window [j - pool/2, j + pool/2] within [0, L-w).
-__global__ void score_pool(const float *__restrict__ raw, const int32_t *__restrict__ lens, int w,
+__global__ void score_pool(const float *__restrict__ raw, const int32_t *__restrict__ lens, ScoreMask mask, int w,
                            int L_cap, int pool, float *__restrict__ scores)
 {
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     const long u = blockIdx.y;
     const int L = lens[u];
-    if (L < w || L > L_cap) return;
+    if (L < w || L > L_cap || mask.skip(u, L, w, L_cap)) return;
     const int nc = L - w;
     if (j >= nc) return;
     const int half = pool / 2;
@@ -198,15 +201,42 @@ __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restr
     scores[u * L_cap + j] = m;
 }
 
-cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
-cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+// The units a masked call scores, in ascending order (one CTA; a ballot scan per
+// 1024 units), and their count.
+__global__ void __launch_bounds__(1024) score_unit_list(const int32_t *__restrict__ lens, ScoreMask mask, int w,
+                                                        int L_cap, int units, int32_t *__restrict__ ulist,
+                                                        int32_t *__restrict__ ucount)
+{
+    __shared__ int warp_n[32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int base = 0;
+    for (int u0 = 0; u0 < units; u0 += blockDim.x) {
+        const int u = u0 + threadIdx.x;
+        const bool take = u < units && !mask.skip(u, lens[u], w, L_cap);
+        const unsigned bal = __ballot_sync(0xffffffffu, take);
+        if (lane == 0) warp_n[wid] = __popc(bal);
+        __syncthreads();
+        int off = base, tot = 0;
+        for (int k = 0; k < nw; ++k) {
+            off += k < wid ? warp_n[k] : 0;
+            tot += warp_n[k];
+        }
+        if (take) ulist[off + __popc(bal & ((1u << lane) - 1u))] = u;
+        base += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *ucount = base;
+}
+
+cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
 bool score_tc_supported(const reco_kv &kv, int w);
 
 template <typename T, int D>
-static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *lens, int w, float c2,
-                              const ScoreWs &ws, unsigned *err, cudaStream_t s)
+static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *lens, ScoreMask mask, int w,
+                              float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s)
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     const int G = kv.H_q / kv.H_kv, R = G * w;
@@ -214,12 +244,12 @@ static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *
     const T *K = (const T *)kv.k;
     int bx = R < 256 ? ((R + 31) / 32) * 32 : 256;
     dim3 g1(nch, (unsigned)units, (R + bx - 1) / bx);
-    score_rowstats_simt<T, D><<<g1, bx, 0, s>>>(q_win, K, lens, w, G, kv.H_q, kv.H_kv, kv.L_cap, R, nch,
-                                                c2, ws.part_m, ws.part_z, err);
+    score_rowstats_simt<T, D><<<g1, bx, 0, s>>>(q_win, K, lens, mask, w, G, kv.H_q, kv.H_kv, kv.L_cap, R,
+                                                nch, c2, ws.part_m, ws.part_z, err);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     long n = units * R;
-    score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, w, kv.L_cap, R, nch, ws.part_m,
+    score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch, ws.part_m,
                                                               ws.part_z, ws.rowb, units);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     size_t smem = ((size_t)R * D + R) * sizeof(float);
@@ -227,7 +257,7 @@ static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *
                              (int)smem);
     if (e != cudaSuccess) return e;
     score_colsum_simt<T, D><<<dim3(nch, (unsigned)units), 128, smem, s>>>(
-        q_win, K, lens, w, G, kv.H_q, kv.H_kv, kv.L_cap, R, c2, ws.rowb, ws.raw);
+        q_win, K, lens, mask, w, G, kv.H_q, kv.H_kv, kv.L_cap, R, c2, ws.rowb, ws.raw);
     return cudaGetLastError();
 }
 
@@ -241,42 +271,46 @@ bool score_shape_supported(const reco_kv &kv, int w)
     return (kv.d == 64 || kv.d == 128) && (R * kv.d + R) <= kSimtMaxQ;
 }
 
-cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, int pool,
-                         float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s)
+cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
+                         int pool, float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s)
 {
     const float c2 = scale * kLog2e;
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const ScoreMask mask{keep, kv.B, kv.H_kv};
     cudaError_t e = cudaSuccess;
     bool used_tc = false;
-    if (kv.dtype == RECO_BF16) {
-        // tensor-core passes: pass 1 -> combine -> pass 2
-        e = launch_score_tc_pass1(kv, q_win, lens, w, c2, ws, err, s, &used_tc);
+    if (kv.dtype == RECO_BF16 && score_tc_supported(kv, w)) {
+        // tensor-core passes: (unit list) -> pass 1 -> combine -> pass 2
+        if (keep) {
+            score_unit_list<<<1, 1024, 0, s>>>(lens, mask, w, kv.L_cap, (int)units, ws.ulist, ws.ucount);
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        }
+        e = launch_score_tc_pass1(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used_tc);
         if (e != cudaSuccess) return e;
         if (used_tc) {
-            const long units = (long)kv.n_layers * kv.B * kv.H_kv;
             const int R = (kv.H_q / kv.H_kv) * w;
             const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
-            score_combine<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, w, kv.L_cap, R, nch, ws.part_m,
-                                                                              ws.part_z, ws.rowb, units);
+            score_combine<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch,
+                                                                              ws.part_m, ws.part_z, ws.rowb, units);
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
             bool used2 = false;
-            e = launch_score_tc_pass2(kv, q_win, lens, w, c2, ws, err, s, &used2);
+            e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used2);
             if (e != cudaSuccess) return e;
             if (!used2) return cudaErrorNotSupported;
         }
     }
     if (!used_tc) {
         if (kv.dtype == RECO_F32)
-            e = kv.d == 64 ? score_simt<float, 64>(kv, (const float *)q_win, lens, w, c2, ws, err, s)
-                           : score_simt<float, 128>(kv, (const float *)q_win, lens, w, c2, ws, err, s);
+            e = kv.d == 64 ? score_simt<float, 64>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s)
+                           : score_simt<float, 128>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s);
         else
             e = kv.d == 64
-                    ? score_simt<__nv_bfloat16, 64>(kv, (const __nv_bfloat16 *)q_win, lens, w, c2, ws, err, s)
-                    : score_simt<__nv_bfloat16, 128>(kv, (const __nv_bfloat16 *)q_win, lens, w, c2, ws, err,
-                                                     s);
+                    ? score_simt<__nv_bfloat16, 64>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws, err, s)
+                    : score_simt<__nv_bfloat16, 128>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws,
+                                                     err, s);
         if (e != cudaSuccess) return e;
     }
-    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
-    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, w, kv.L_cap,
+    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,
                                                                             pool, scores);
     return cudaGetLastError();
 }

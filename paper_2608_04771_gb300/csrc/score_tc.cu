@@ -127,18 +127,20 @@ __device__ __forceinline__ bool wait_or_flag(uint32_t bar, uint32_t parity, vola
 
 // ---------------------------------------------------------------- work items
 // A CTA walks a contiguous range of (unit, 2048-key chunk) items in unit order, so its
-// window queries change only when the unit does.
+// window queries change only when the unit does.  Item i covers unit i / n_chunks, or,
+// when a unit list is given (a masked call), unit ulist[i / n_chunks]: the ranges are
+// then cut from the scored units only, which keeps the CTAs evenly loaded.
 struct ChunkItem {
     long u;
     int chunk, L, j0, j1, ntiles;
     bool valid;  // the unit's length is in range
 };
 
-__device__ __forceinline__ ChunkItem chunk_item(int i, int n_chunks, const int32_t *lens, int w, int L_cap,
-                                               bool candidates_only, int tile)
+__device__ __forceinline__ ChunkItem chunk_item(int i, int n_chunks, const int32_t *ulist, const int32_t *lens,
+                                               int w, int L_cap, bool candidates_only, int tile)
 {
     ChunkItem it;
-    it.u = i / n_chunks;
+    it.u = ulist ? ulist[i / n_chunks] : i / n_chunks;
     it.chunk = i % n_chunks;
     it.L = lens[it.u];
     it.valid = it.L >= w && it.L <= L_cap;
@@ -154,7 +156,8 @@ template <int D, int N, int MT>
 __global__ void __launch_bounds__(128 + 128 * MT, 1)
     score_rowstats_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R,
-                      int n_chunks, int n_items, float c2, float *__restrict__ part_m, float *__restrict__ part_z,
+                      int n_chunks, int n_items, const int32_t *__restrict__ ulist, const int32_t *__restrict__ ucount,
+                      float c2, float *__restrict__ part_m, float *__restrict__ part_z,
                       unsigned *err)
 {
     constexpr int HALVES = D / 64;
@@ -170,8 +173,9 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
     __shared__ int abort_sh;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int i_begin = (int)((long long)blockIdx.x * n_items / gridDim.x);
-    const int i_end = (int)((long long)(blockIdx.x + 1) * n_items / gridDim.x);
+    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
+    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
     const uint32_t raw0 = smem_addr(smem_raw);
     const uint32_t base = (raw0 + 1023u) & ~1023u;
     const uint32_t Qs = base;                                  // MT x HALVES x QBOX
@@ -206,7 +210,7 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
-                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+                const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, false, N);
                 if (it.ntiles == 0) continue;
                 if (it.u != prev_u) {
                     if (nq > 0 && !wait_or_flag(smem_addr(&bar_qempty), (nq - 1) & 1, abort_flag, err)) break;
@@ -239,7 +243,7 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
-                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+                const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, false, N);
                 if (it.ntiles == 0) continue;
                 if (it.u != prev_u) {
                     if (nq > 0) tc_commit(smem_addr(&bar_qempty));  // queries free once prior MMAs land
@@ -276,7 +280,7 @@ __global__ void __launch_bounds__(128 + 128 * MT, 1)
         const int t_row = r % w;
         int gt = 0;
         for (int i = i_begin; i < i_end; ++i) {
-            const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, false, N);
+            const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, false, N);
             if (!it.valid) {
                 if (it.chunk == 0 && r == 0) raise_error(err, ERR_LEN);
                 continue;
@@ -349,7 +353,8 @@ template <int D>
 __global__ void __launch_bounds__(128 + 256, 1)
     score_colsum_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R, int NQ,
-                    int n_chunks, int n_items, float c2, const float *__restrict__ rowb, float *__restrict__ raw,
+                    int n_chunks, int n_items, const int32_t *__restrict__ ulist, const int32_t *__restrict__ ucount,
+                    float c2, const float *__restrict__ rowb, float *__restrict__ raw,
                     unsigned *err)
 {
     constexpr int HALVES = D / 64;
@@ -364,8 +369,9 @@ __global__ void __launch_bounds__(128 + 256, 1)
     __shared__ float bsh[8][kTcMaxR];  // per epilogue warp: row normalisers of its current unit
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int i_begin = (int)((long long)blockIdx.x * n_items / gridDim.x);
-    const int i_end = (int)((long long)(blockIdx.x + 1) * n_items / gridDim.x);
+    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
+    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
     const bool split_cols = NQ > 256;
     const int NBUF = split_cols ? 1 : 2;
     const int nmma = split_cols ? 2 : 1;
@@ -407,7 +413,7 @@ __global__ void __launch_bounds__(128 + 256, 1)
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
-                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+                const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, true, 128);
                 if (it.ntiles == 0) continue;
                 if (it.u != prev_u) {
                     if (nq > 0 && !wait_or_flag(smem_addr(&bar_qempty), (nq - 1) & 1, abort_flag, err)) break;
@@ -440,7 +446,7 @@ __global__ void __launch_bounds__(128 + 256, 1)
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
-                const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+                const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, true, 128);
                 if (it.ntiles == 0) continue;
                 if (it.u != prev_u) {
                     if (nq > 0) tc_commit(smem_addr(&bar_qempty));
@@ -481,7 +487,7 @@ __global__ void __launch_bounds__(128 + 256, 1)
         int gt = 0;
         long prev_u = -1;
         for (int i = i_begin; i < i_end; ++i) {
-            const ChunkItem it = chunk_item(i, n_chunks, lens, w, L_cap, true, 128);
+            const ChunkItem it = chunk_item(i, n_chunks, ulist, lens, w, L_cap, true, 128);
             if (it.ntiles == 0) continue;
             if (it.u != prev_u) {  // this unit's row normalisers (warp-private copy)
                 __syncwarp();
@@ -555,8 +561,8 @@ bool score_tc_supported(const reco_kv &kv, int w)
 }
 
 template <int D, int N, int MT>
-static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                             const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                             float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     const int R = (kv.H_q / kv.H_kv) * w;
@@ -575,37 +581,39 @@ static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t
     const int n_items = (int)(units * nch);
     const int grid = min(n_items, device_sm_count());
     score_rowstats_tc<D, N, MT><<<grid, 128 + 128 * MT, smem, s>>>(mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q,
-                                                                  kv.H_kv, kv.L_cap, R, nch, n_items, c2,
-                                                                  ws.part_m, ws.part_z, err);
+                                                                  kv.H_kv, kv.L_cap, R, nch, n_items,
+                                                                  masked ? ws.ulist : nullptr,
+                                                                  masked ? ws.ucount : nullptr, c2, ws.part_m,
+                                                                  ws.part_z, err);
     *ok = true;
     return cudaGetLastError();
 }
 
 template <int D>
-static cudaError_t pass1_by_mt(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                               const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+static cudaError_t pass1_by_mt(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                               float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
 {
     const int MT = ((kv.H_q / kv.H_kv) * w + 127) / 128;
     switch (MT) {
-    case 1: return run_pass1<D, 128, 1>(kv, q_win, lens, w, c2, ws, err, s, ok);
-    case 2: return run_pass1<D, 128, 2>(kv, q_win, lens, w, c2, ws, err, s, ok);
-    case 3: return run_pass1<D, 64, 3>(kv, q_win, lens, w, c2, ws, err, s, ok);
-    default: return run_pass1<D, 64, 4>(kv, q_win, lens, w, c2, ws, err, s, ok);
+    case 1: return run_pass1<D, 128, 1>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
+    case 2: return run_pass1<D, 128, 2>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
+    case 3: return run_pass1<D, 64, 3>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
+    default: return run_pass1<D, 64, 4>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
     }
 }
 
-cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
 {
     *used = false;
     if (!score_tc_supported(kv, w)) return cudaSuccess;
-    return kv.d == 128 ? pass1_by_mt<128>(kv, q_win, lens, w, c2, ws, err, s, used)
-                       : pass1_by_mt<64>(kv, q_win, lens, w, c2, ws, err, s, used);
+    return kv.d == 128 ? pass1_by_mt<128>(kv, q_win, lens, masked, w, c2, ws, err, s, used)
+                       : pass1_by_mt<64>(kv, q_win, lens, masked, w, c2, ws, err, s, used);
 }
 
 template <int D>
-static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                             const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                             float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     const int R = (kv.H_q / kv.H_kv) * w;
@@ -628,18 +636,19 @@ static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t
     const int n_items = (int)(units * nch);
     const int grid = min(n_items, device_sm_count());
     score_colsum_tc<D><<<grid, 128 + 256, smem, s>>>(mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R,
-                                                     NQ, nch, n_items, c2, ws.rowb, ws.raw, err);
+                                                     NQ, nch, n_items, masked ? ws.ulist : nullptr,
+                                                     masked ? ws.ucount : nullptr, c2, ws.rowb, ws.raw, err);
     *ok = true;
     return cudaGetLastError();
 }
 
-cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, int w, float c2,
-                                  const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
+                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
 {
     *used = false;
     if (!score_tc_supported(kv, w)) return cudaSuccess;
-    return kv.d == 128 ? run_pass2<128>(kv, q_win, lens, w, c2, ws, err, s, used)
-                       : run_pass2<64>(kv, q_win, lens, w, c2, ws, err, s, used);
+    return kv.d == 128 ? run_pass2<128>(kv, q_win, lens, masked, w, c2, ws, err, s, used)
+                       : run_pass2<64>(kv, q_win, lens, masked, w, c2, ws, err, s, used);
 }
 
 }  // namespace reco

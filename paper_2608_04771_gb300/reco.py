@@ -62,7 +62,7 @@ def lib():
     L.reco_last_error.argtypes = []
     L.reco_last_error.restype = ctypes.c_char_p
     L.reco_check.argtypes = [vp]
-    L.reco_score_cache.argtypes = [kvp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
+    L.reco_score_cache.argtypes = [kvp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
@@ -149,9 +149,10 @@ def reco_check(stream=None):
 
 
 # ---------------------------------------------------------------- device calls
-def reco_score_cache(kv: reco_kv, q_win, lens, w: int, pool_kernel: int, scale: float, scores, ws,
+def reco_score_cache(kv: reco_kv, q_win, lens, w: int, pool_kernel: int, scale: float, scores, ws, keep=None,
                      stream=None):
-    _ok(lib().reco_score_cache(ctypes.byref(kv), _ptr(q_win), _ptr(lens), int(w), int(pool_kernel),
+    """keep (optional [B] int32): skip the units of sequences with keep[b] >= lens."""
+    _ok(lib().reco_score_cache(ctypes.byref(kv), _ptr(q_win), _ptr(lens), _ptr(keep), int(w), int(pool_kernel),
                                float(scale), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
 
 

@@ -10,7 +10,7 @@ When a sequence completes a step it receives a reward v_i (Sec. 3.1), and
     (L - L_{i-1} >= S, Sec. 3.2; L_0 = the prompt; S = 0 compresses at every
     step boundary) it is compressed to m_i = lambda_i * L (Eq. 1-2, Sec. 3.2) --
     all sequences are passed to one scoring/selection call, the others with
-    keep = L, which leaves them untouched;
+    keep = L, which skips their scoring and leaves them untouched;
   * if v_{i-1} >= tau_h and v_i >= tau_h, the answer probe runs (Eq. 5-6) and a
     sequence that passes PPL <= tau_p stops and leaves the batch.
 Budget base L (the paper is silent on repeated compression): reading "A" uses the
@@ -331,8 +331,9 @@ class Trace:
             if info:
                 q_win = self._sel(self.window_queries(t))
                 keep_dev = _to_device(keep, torch.int32, self.device)
+                # only the sequences compressed now are scored (keep == L skips the rest)
                 reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
-                                      self.ws_score)
+                                      self.ws_score, keep=keep_dev)
                 reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
                                          self.ws_select)
             if on_boundary:

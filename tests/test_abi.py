@@ -103,13 +103,13 @@ def test_device_calls_validate_before_launch(L):
     kv = _kv()
     vp = ctypes.c_void_p
     ws = vp(256 * 1000)
-    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 0, 7, 0.1, vp(16), ws, 10, None)
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), None, 0, 7, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
-    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 16, 4, 0.1, vp(16), ws, 10, None)
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), None, 16, 4, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"pool_kernel" in L.reco_last_error()
-    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
+    st = L.reco_score_cache(ctypes.byref(kv), vp(16), vp(16), None, 16, 7, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
-    st = L.reco_score_cache(ctypes.byref(_kv(k=17)), vp(16), vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
+    st = L.reco_score_cache(ctypes.byref(_kv(k=17)), vp(16), vp(16), None, 16, 7, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
     st = L.reco_select_compact(ctypes.byref(kv), None, vp(16), vp(16), 16, None, ws, 10, None)
     assert st == reco.RECO_EINVAL

@@ -44,5 +44,5 @@ def test_window_rows_beyond_both_scoring_paths_are_rejected():
     K, V = W.make_cache(wl, "cuda", canary=False)
     kv = reco.make_kv(K, V, wl.h_q)
     st = reco.lib().reco_score_cache(ctypes.byref(kv), ctypes.c_void_p(K.data_ptr()), ctypes.c_void_p(16),
-                                     wl.w, 7, 0.1, ctypes.c_void_p(16), ctypes.c_void_p(256 * 4096), 1 << 40, None)
+                                     None, wl.w, 7, 0.1, ctypes.c_void_p(16), ctypes.c_void_p(256 * 4096), 1 << 40, None)
     assert st == reco.RECO_EUNSUPPORTED
