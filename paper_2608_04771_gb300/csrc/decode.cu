@@ -4,7 +4,8 @@
 // bf16 path (decode_tma): a persistent split-K flash-decode, one CTA of 8 warps per
 // SM.  Every CTA first builds the same work plan from lens: a key-chunk length C
 // chosen so the total number of (unit, chunk) items is several per warp, and the
-// prefix sum of chunks per unit.  Each warp then takes items from an atomic counter.
+// prefix sum of chunks per unit.  Each warp's first two items are dealt out
+// statically, round-robin over the CTAs; the rest come from an atomic counter.
 // An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
 // (128-byte swizzled 16 x 64 tiles of K and V) into the warp's 3-stage ring and the
 // warp waits on the stage's mbarrier (bounded).  QK^T and PV run on mma.sync
@@ -215,6 +216,8 @@ constexpr int kDecodeStages = 3;      // ring stages per warp
 constexpr int kItemsPerWarp = 4;      // target work items per warp (fewer, larger items pay less per-item cost)
 constexpr int kMaxTmaUnits = 3072;    // two plan entries per unit kept in shared memory
 constexpr long long kSpinLimit = 1LL << 24;  // bounded mbarrier waits (about a second)
+constexpr float kLazyLog2 = 8.f;             // output rescale threshold (log2 units)
+constexpr int kDecodeMinChunk = 256;         // shortest full chunk (keys): a split costs a merge
 
 template <int D> struct TmaLayout {
     static constexpr int HALVES = D / 64;             // 128-byte boxes per row
@@ -250,6 +253,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
     const uint32_t my_ring = ring0 + (uint32_t)wid * S * STAGE;
+    if (tid == 0) {  // fetch both tensor-map descriptors while the plan is built
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    }
     if (lane == 0) {
         for (int s2 = 0; s2 < S; ++s2) mbar_init((uint32_t)__cvta_generic_to_shared(&bars[wid][s2]), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -272,11 +279,23 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // stage the lengths in the (still idle) ring memory with one coalesced sweep; the
     // plan below reads them from there (the ring is first written by TMA after the plan)
     int *len_sm = reinterpret_cast<int *>(smem_raw + (ring0 - raw0));
-    for (int u = tid; u < units; u += blockDim.x) {
-        const int L = a.lens[u];
-        const bool ok = unit_ok(L, a.L_cap, a.append);
-        if (!ok && blockIdx.x == 0) raise_error(a.err, (a.append && L == a.L_cap) ? ERR_ROOM : ERR_LEN);
-        len_sm[u] = ok ? L + a.append : 0;
+    for (int u0 = 0; u0 < units; u0 += 8 * (int)blockDim.x) {
+        int Lr[8];  // all loads of the batch in flight before any store or error report
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int u = u0 + k * (int)blockDim.x + tid;
+            Lr[k] = u < units ? __ldcg(a.lens + u) : 0;
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int u = u0 + k * (int)blockDim.x + tid;
+            if (u < units) {
+                const bool ok = unit_ok(Lr[k], a.L_cap, a.append);
+                if (!ok && blockIdx.x == 0)
+                    raise_error(a.err, (a.append && Lr[k] == a.L_cap) ? ERR_ROOM : ERR_LEN);
+                len_sm[u] = ok ? Lr[k] + a.append : 0;
+            }
+        }
     }
     __syncthreads();
     long long tot = 0;
@@ -291,7 +310,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     const long long target = min((long long)kDecodeMaxTarget, (long long)kItemsPerWarp * total_warps);
     long long Cl = (tot + target - 1) / target;
     Cl = ((Cl + 63) / 64) * 64;
-    if (Cl < 256) Cl = 256;
+    if (Cl < kDecodeMinChunk) Cl = kDecodeMinChunk;
     const int C = (int)Cl;
     int my_f = 0, my_t = 0;
     for (int u = u_lo; u < u_hi; ++u) {
@@ -373,12 +392,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         it.nblk = (it.k1 - it.k0 + 15) / 16;
         return it;
     };
-    auto grab = [&]() {
+    // Items 0 .. 2*total_warps-1 are dealt out statically (two per warp);
+    // the counter hands out the rest.  A warp takes its counter ticket one item ahead
+    // (issued when an item starts, read when it ends) so the atomic's latency is hidden.
+    auto ticket = [&]() {
         int d = 0;
         if (lane == 0) d = atomicAdd(&a.counters[0], 1);
-        d = __shfl_sync(0xffffffffu, d, 0);
-        return meta(d);
+        return d;
     };
+    auto redeem = [&](int d) { return meta(2 * total_warps + __shfl_sync(0xffffffffu, d, 0)); };
 
     // Q fragments of an item (rows g < G), head dim permuted to match the K chunks:
     // k-step j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
@@ -404,10 +426,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // item into the next one (grabbed one item ahead) so no refill bubble opens between
     // items; the warp consumes blocks in issue order.
     uint32_t issued = 0, consumed = 0;
-    Item cur = grab();
-    Item nxt = cur.nblk >= 0 ? grab() : cur;
+    // static deal interleaved across CTAs (warp wid of every CTA before warp wid+1 of
+    // any): a partial round then spreads evenly over the SMs, whose warps share one
+    // TMA unit and one L2 port
+    const int gw = wid * (int)gridDim.x + (int)blockIdx.x;
+    Item cur = meta(gw);
     uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
     if (cur.nblk >= 0) load_q(cur, qa_n);
+    Item nxt = cur.nblk >= 0 ? meta(gw + total_warps) : cur;
+    int tk = 0;  // counter ticket for the item after nxt
     Item pit = cur;  // item the producer is issuing from
     int pblk = 0;
     bool p_on_next = false;
@@ -451,13 +478,19 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         const long qrow0 = lb * a.Hq + (long)h * G;
         const int row0 = u * a.L_cap;  // first tensor-map row of this unit
 
+        // start this item's copies before the wait on its query registers below
+        __syncwarp();
+        while (issued - consumed < (uint32_t)S && can_issue()) issue();
         uint32_t qa[D / 16][2];
 #pragma unroll
         for (int j = 0; j < D / 16; ++j) {
             qa[j][0] = qa_n[j][0];
             qa[j][1] = qa_n[j][1];
         }
-        if (nxt.nblk >= 0) load_q(nxt, qa_n);  // the next item's queries load while this one streams
+        if (nxt.nblk >= 0) {
+            load_q(nxt, qa_n);  // the next item's queries load while this one streams
+            tk = ticket();
+        }
         float o[MT][4];
 #pragma unroll
         for (int t = 0; t < MT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
@@ -496,7 +529,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 }
                 __syncwarp();
             }
+            // four accumulators (keys 0-7 / 8-15, even / odd k-steps): dependent MMA chains
+            // of D/32 instead of D/16
             float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+            float t0[4] = {0.f, 0.f, 0.f, 0.f}, t1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int hh = 0; hh < HALVES; ++hh)
 #pragma unroll
@@ -506,9 +542,14 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                     const int j = 4 * hh + 2 * e;
                     mma_bf16(s0, qa[j][0], 0u, qa[j][1], 0u, ka.x, ka.y);
                     mma_bf16(s1, qa[j][0], 0u, qa[j][1], 0u, kc.x, kc.y);
-                    mma_bf16(s0, qa[j + 1][0], 0u, qa[j + 1][1], 0u, ka.z, ka.w);
-                    mma_bf16(s1, qa[j + 1][0], 0u, qa[j + 1][1], 0u, kc.z, kc.w);
+                    mma_bf16(t0, qa[j + 1][0], 0u, qa[j + 1][1], 0u, ka.z, ka.w);
+                    mma_bf16(t1, qa[j + 1][0], 0u, qa[j + 1][1], 0u, kc.z, kc.w);
                 }
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                s0[i] += t0[i];
+                s1[i] += t1[i];
+            }
             // scores of query g for keys kb+2c, kb+2c+1, kb+8+2c, kb+9+2c
             const int kA = kb + 2 * c, kB = kb + 8 + 2 * c;
             const float x0 = (kA < k1) ? s0[0] * a.c2 : -INFINITY;
@@ -518,22 +559,31 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             float mb = fmaxf(fmaxf(x0, x1), fmaxf(x2, x3));
             mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, 1));
             mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, 2));
-            const float mn = fmaxf(m, mb);
-            const float base = (mn == -INFINITY) ? 0.f : mn;
-            const float alpha = fast_exp2(m - base);
+            // Lazy rescale: a row's reference max m moves only when a block max exceeds it
+            // by more than 2^kLazyLog2, so probabilities against a stale m stay <= 2^8
+            // (exact in fp32, and the bf16 hi + lo split keeps 16 bits of them); the
+            // output rescale below then runs on few blocks.  m, l and o stay consistent, so
+            // o / l and lse = m + log2 l are the same quantities as with an exact max.
+            const bool grow = mb > m + kLazyLog2;
+            if (__any_sync(0xffffffffu, grow)) {
+                const float mn = grow ? mb : m;
+                const float alpha = grow ? fast_exp2(m - mn) : 1.f;  // m = -inf gives 0
+                l *= alpha;
+                m = mn;
+                const float a0 = __shfl_sync(0xffffffffu, alpha, (2 * c) * 4);
+                const float a1 = __shfl_sync(0xffffffffu, alpha, (2 * c + 1) * 4);
+#pragma unroll
+                for (int t = 0; t < MT; ++t) {
+                    o[t][0] *= a0;
+                    o[t][1] *= a1;
+                    o[t][2] *= a0;
+                    o[t][3] *= a1;
+                }
+            }
+            const float base = (m == -INFINITY) ? 0.f : m;
             const float p0 = fast_exp2(x0 - base), p1 = fast_exp2(x1 - base);
             const float p2 = fast_exp2(x2 - base), p3 = fast_exp2(x3 - base);
-            l = l * alpha + ((p0 + p1) + (p2 + p3));
-            m = mn;
-            const float a0 = __shfl_sync(0xffffffffu, alpha, (2 * c) * 4);
-            const float a1 = __shfl_sync(0xffffffffu, alpha, (2 * c + 1) * 4);
-#pragma unroll
-            for (int t = 0; t < MT; ++t) {
-                o[t][0] *= a0;
-                o[t][1] *= a1;
-                o[t][2] *= a0;
-                o[t][3] *= a1;
-            }
+            l += (p0 + p1) + (p2 + p3);
             // P enters the PV product as bf16 hi + lo parts (two MMAs), which keeps about
             // 16 significant bits of each probability instead of 8.
             uint32_t ph0, ph1, pl0, pl1;
@@ -680,7 +730,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         // advance: the producer may already be streaming the next item's blocks
         cur = nxt;
-        nxt = cur.nblk >= 0 ? grab() : cur;
+        nxt = cur.nblk >= 0 ? redeem(tk) : cur;
         if (p_on_next) {
             p_on_next = false;
         } else {
@@ -696,9 +746,21 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     done = __shfl_sync(0xffffffffu, done, 0);
     __syncwarp();
     if (done == total_warps - 1 && a.append) {
-        for (int u = lane; u < units; u += 32) {
-            const int le = eff_len(u);
-            if (le >= 0) a.lens[u] = le;
+        // 16 independent loads per lane in flight before any store: a few L2 round trips
+        // for the whole grid instead of one per 32 units
+        constexpr int BATCH = 16;
+        for (int u0 = 0; u0 < units; u0 += 32 * BATCH) {
+            int L[BATCH];
+#pragma unroll
+            for (int k = 0; k < BATCH; ++k) {
+                const int u = u0 + 32 * k + lane;
+                L[k] = u < units ? __ldcg(a.lens + u) : -1;
+            }
+#pragma unroll
+            for (int k = 0; k < BATCH; ++k) {
+                const int u = u0 + 32 * k + lane;
+                if (u < units && unit_ok(L[k], a.L_cap, a.append)) a.lens[u] = L[k] + 1;
+            }
         }
     }
 }

@@ -51,9 +51,35 @@ def _pack(parts, out=None):
     return buf, views
 
 
-def _to_device(values, dtype, device):
-    """Host list -> device tensor through pinned memory, without blocking the host."""
-    return torch.tensor(values, dtype=dtype).pin_memory().to(device, non_blocking=True)
+class _Staging:
+    """Small host -> device copies (keep counts, rewards) through a ring of pinned host
+    slots.  A slot is written again only after the copy that last read it has completed
+    (one event per slot), so the host never blocks on a busy GPU queue and never
+    allocates pinned memory in the loop.  A device slot is reused only by a later copy on
+    the same stream, after every kernel that read it."""
+
+    def __init__(self, n_max: int, device, n_slots: int = 64):
+        self.host = torch.zeros((n_slots, n_max), dtype=torch.int32).pin_memory()
+        self.host_np = self.host.numpy()
+        self.dev = torch.zeros((n_slots, n_max), dtype=torch.int32, device=device)
+        self.events = [torch.cuda.Event() for _ in range(n_slots)]
+        self.used = [False] * n_slots
+        self.next = 0
+
+    def put(self, values, dtype, out=None) -> torch.Tensor:
+        """Copy `values` to the device (into `out` if given, else a ring slot)."""
+        i = self.next
+        self.next = (i + 1) % len(self.events)
+        if self.used[i]:
+            self.events[i].synchronize()
+        n = len(values)
+        self.host_np[i, :n] = np.asarray(values, dtype=np.int32 if dtype == torch.int32 else np.float32).view(np.int32)
+        src = self.host[i, :n].view(dtype)
+        dst = out if out is not None else self.dev[i, :n].view(dtype)
+        dst.copy_(src, non_blocking=True)
+        self.events[i].record()
+        self.used[i] = True
+        return dst
 
 
 @dataclass
@@ -126,6 +152,7 @@ class Trace:
         self.step_idx = [0] * spec.batch
         self.out_dtype = out_dtype
         self.ids = torch.from_numpy(W.make_reflection_ids(wl)).to(device) if wl.vocab else None
+        self.staging = _Staging(spec.batch, device)
         self._pool = None
         if input_pool:
             self._pool = [(self._token_inputs(t), self._window_queries(t) if t < 8 else None,
@@ -239,7 +266,7 @@ class Trace:
         self.g_logits = views[3] if self.ids is not None else None
         self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
         self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
-        self.g_rw = _to_device([self.current_reward(s) for s in self.active], torch.float32, dev)
+        self.g_rw = self.staging.put([self.current_reward(s) for s in self.active], torch.float32).clone()
         # one call outside the capture, without an append (cache and lens stay as they are)
         reco.reco_decode_attn(self.kv, self.g_q, None, None, self.lens_dev, wl.scale(), self.g_out, self.g_lse,
                               self.ws_decode)
@@ -280,7 +307,7 @@ class Trace:
         logits = None
         if self.ids is not None:
             logits = self.active_logits(t)
-            rw = _to_device([self.current_reward(s) for s in self.active], torch.float32, self.device)
+            rw = self.staging.put([self.current_reward(s) for s in self.active], torch.float32)
             reco.reco_reflect_penalty(logits, self.ids, rw, wl.tau_l, wl.tau_h, wl.beta)
         return out, lse, logits
 
@@ -330,7 +357,7 @@ class Trace:
             q_win = None
             if info:
                 q_win = self._sel(self.window_queries(t))
-                keep_dev = _to_device(keep, torch.int32, self.device)
+                keep_dev = self.staging.put(keep, torch.int32)
                 # only the sequences compressed now are scored (keep == L skips the rest)
                 reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
                                       self.ws_score, keep=keep_dev)
@@ -357,6 +384,5 @@ class Trace:
             if gone:
                 self._drop(gone)
             elif self.use_graph and self.graph is not None:
-                self.g_rw.copy_(_to_device([self.current_reward(s) for s in self.active], torch.float32,
-                                           self.device))
+                self.staging.put([self.current_reward(s) for s in self.active], torch.float32, out=self.g_rw)
         return ev
