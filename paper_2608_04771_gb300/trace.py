@@ -63,6 +63,7 @@ class _Staging:
         self.host_np = self.host.numpy()
         self.dev = torch.zeros((n_slots, n_max), dtype=torch.int32, device=device)
         self.events = [torch.cuda.Event() for _ in range(n_slots)]
+        self.stream = torch.cuda.current_stream(device)
         self.used = [False] * n_slots
         self.next = 0
 
@@ -77,7 +78,7 @@ class _Staging:
         src = self.host[i, :n].view(dtype)
         dst = out if out is not None else self.dev[i, :n].view(dtype)
         dst.copy_(src, non_blocking=True)
-        self.events[i].record()
+        self.events[i].record(self.stream)
         self.used[i] = True
         return dst
 
@@ -154,9 +155,22 @@ class Trace:
         self.ids = torch.from_numpy(W.make_reflection_ids(wl)).to(device) if wl.vocab else None
         self.staging = _Staging(spec.batch, device)
         self._pool = None
+        self._answers = {}
         if input_pool:
-            self._pool = [(self._token_inputs(t), self._window_queries(t) if t < 8 else None,
-                           self._token_logits(t) if wl.vocab else None) for t in range(input_pool)]
+            # every slot's inputs stacked on a leading slot axis: [P, Ly, B, ...], [P, B, V]
+            ins = [self._token_inputs(t) for t in range(input_pool)]
+            self._pool = (torch.stack([x[0] for x in ins]), torch.stack([x[1] for x in ins]),
+                          torch.stack([x[2] for x in ins]),
+                          torch.stack([self._token_logits(t) for t in range(input_pool)]) if wl.vocab else None,
+                          torch.stack([self._window_queries(t) for t in range(8)]))
+            del ins
+            # the answers of every probe the rewards can trigger, drawn before the loop runs
+            for sq in range(spec.batch):
+                r = np.asarray(self.rewards[sq], np.float32)
+                for k in range(1, len(r)):
+                    t = int(self.ends[sq][k])
+                    if t < spec.generated and r[k - 1] >= np.float32(wl.tau_h) and r[k] >= np.float32(wl.tau_h):
+                        self._answers[(t, sq)] = self._answer(t, sq)
         self._rebuild()
 
     # ---------------------------------------------------------------- inputs
@@ -172,16 +186,23 @@ class Trace:
 
     def token_inputs(self, t: int):
         """q [Ly, B, Hq, d], k_new / v_new [Ly, B, Hkv, d] for token t, full batch."""
-        return self._pool[t % self.input_pool][0] if self._pool else self._token_inputs(t)
+        if self._pool:
+            i = t % self.input_pool
+            return self._pool[0][i], self._pool[1][i], self._pool[2][i]
+        return self._token_inputs(t)
 
     def window_queries(self, t: int):
-        return self._pool[t % 8][1] if self._pool else self._window_queries(t)
+        return self._pool[4][t % 8] if self._pool else self._window_queries(t)
 
     def token_logits(self, t: int):
-        return self._pool[t % self.input_pool][2].clone() if self._pool else self._token_logits(t)
+        return self._pool[3][t % self.input_pool].clone() if self._pool else self._token_logits(t)
 
     def answer(self, t: int, seq: int):
         """Answer logits / tokens of a probe of sequence `seq` at token t (confident on even probes)."""
+        got = self._answers.get((t, seq))
+        return got if got is not None else self._answer(t, seq)
+
+    def _answer(self, t: int, seq: int):
         wl = self.wl.reduced(batch=1, seed=self.spec.seed * 7919 + t * 31 + seq)
         z, tok = W.make_answer(wl, self.device)
         if (t + seq) % 2:  # every other probe is not confident
@@ -198,29 +219,49 @@ class Trace:
     def active_inputs(self, t: int):
         """Token t's q, k_new, v_new for the active sequences."""
         if self._apool is not None:
-            return self._apool[t % self.input_pool][1]
+            return tuple(self._slot_view(t % self.input_pool, k) for k in range(3))
         q, kn, vn = self._token_inputs(t)
         return self._sel(q), self._sel(kn), self._sel(vn)
 
     def active_logits(self, t: int):
         """A fresh copy of token t's logits rows of the active sequences."""
         if self._apool is not None:
-            return self._apool[t % self.input_pool][2].clone()
+            return self._slot_view(t % self.input_pool, 3).clone()
         return self._sel(self._token_logits(t), 0)
+
+    def active_window_queries(self, t: int):
+        if self._apool is not None:
+            return self._awin[t % 8]
+        return self._sel(self._window_queries(t))
 
     # ---------------------------------------------------------------- plumbing
     def _active_pool(self):
-        """The input pool restricted to the active sequences.  Each slot's q | k_new | v_new
-        | logits are packed into one byte buffer laid out like the captured graph's static
-        inputs, so a token's inputs arrive in a single copy."""
+        """The input pool restricted to the active sequences (one gather per input over all
+        slots).  Slot i's q | k_new | v_new | logits are packed in row i of one byte matrix,
+        laid out like the captured graph's static inputs (each part 256-byte aligned), so a
+        token's inputs arrive in a single copy."""
         if not self._pool:
+            self._awin = None
             return None
-        apool = []
-        for (q, kn, vn), _, z in self._pool:
-            parts = [self._sel(q), self._sel(kn), self._sel(vn)] + ([] if z is None else [self._sel(z, 0)])
-            packed, views = _pack(parts)
-            apool.append((packed, tuple(views[:3]), views[3] if z is not None else None))
-        return apool
+        P = self.input_pool
+        Q, KN, VN, Z, WQ = self._pool
+        sel = (lambda x, d: x) if self._full_batch() else (lambda x, d: x.index_select(d, self.idx_dev))
+        parts = [sel(Q, 2), sel(KN, 2), sel(VN, 2)] + ([] if Z is None else [sel(Z, 1)])
+        self._slot_meta, cols, off = [], [], 0
+        for x in parts:
+            nb = x[0].numel() * x.element_size()
+            cols.append(x.reshape(P, -1).contiguous().view(torch.uint8))
+            pad = (nb + 255) // 256 * 256 - nb
+            if pad:
+                cols.append(torch.zeros((P, pad), dtype=torch.uint8, device=x.device))
+            self._slot_meta.append((off, nb, x.dtype, tuple(x.shape[1:])))
+            off += nb + pad
+        self._awin = sel(WQ, 2).contiguous()
+        return torch.cat(cols, dim=1)
+
+    def _slot_view(self, i: int, k: int):
+        off, nb, dt, shape = self._slot_meta[k]
+        return self._apool[i, off:off + nb].view(dt).view(shape)
 
     def _rebuild(self):
         wl = self.wl
@@ -290,7 +331,7 @@ class Trace:
             if self.graph is None:
                 self._capture()
             if self._apool is not None:
-                self.g_in.copy_(self._apool[t % self.input_pool][0])
+                self.g_in.copy_(self._apool[t % self.input_pool])
             else:
                 q, kn, vn = self.active_inputs(t)
                 self.g_q.copy_(q)
@@ -356,7 +397,7 @@ class Trace:
                 ev.compressions += 1
             q_win = None
             if info:
-                q_win = self._sel(self.window_queries(t))
+                q_win = self.active_window_queries(t)
                 keep_dev = self.staging.put(keep, torch.int32)
                 # only the sequences compressed now are scored (keep == L skips the rest)
                 reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
