@@ -153,7 +153,7 @@ class Trace:
         self.step_idx = [0] * spec.batch
         self.out_dtype = out_dtype
         self.ids = torch.from_numpy(W.make_reflection_ids(wl)).to(device) if wl.vocab else None
-        self.staging = _Staging(spec.batch, device)
+        self.staging = _Staging(2 * spec.batch, device)
         self._pool = None
         self._answers = {}
         if input_pool:
@@ -292,8 +292,10 @@ class Trace:
         self.last_comp = [self.last_comp[i] for i in keep_pos]
         self._rebuild()
 
-    def _capture(self):
-        """Static input/output buffers and one CUDA graph of a token's decode + penalty."""
+    def _capture(self, t: int):
+        """Static input/output buffers and one CUDA graph of a token's decode + penalty.
+        With an input pool the graph also gathers its token's inputs (slot slot_dev of
+        the packed pool) and advances slot_dev, so a token costs the host one launch."""
         wl, dev, B = self.wl, self.device, len(self.active)
         shapes = [((wl.layers, B, wl.h_q, wl.d), wl.torch_dtype), ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype),
                   ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype)]
@@ -307,18 +309,35 @@ class Trace:
         self.g_logits = views[3] if self.ids is not None else None
         self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
         self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
-        self.g_rw = self.staging.put([self.current_reward(s) for s in self.active], torch.float32).clone()
+        # keep counts (row 0) and current rewards (row 1, float32 bits): one upload per boundary
+        self.g_small = torch.zeros((2, B), dtype=torch.int32, device=dev)
+        self.g_rw = self.g_small[1].view(torch.float32)
+        self._put_small(list(self.lens))
+        self.g_slot = torch.zeros(1, dtype=torch.long, device=dev)
         # one call outside the capture, without an append (cache and lens stay as they are)
         reco.reco_decode_attn(self.kv, self.g_q, None, None, self.lens_dev, wl.scale(), self.g_out, self.g_lse,
                               self.ws_decode)
         torch.cuda.synchronize()
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="relaxed"):
+            if self._apool is not None:
+                # 8-byte elements: every part is a multiple of 256 bytes
+                torch.index_select(self._apool.view(torch.int64), 0, self.g_slot,
+                                   out=self.g_in.view(torch.int64).view(1, -1))
             reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
                                   self.g_lse, self.ws_decode)
             if self.g_logits is not None:
                 reco.reco_reflect_penalty(self.g_logits, self.ids, self.g_rw, wl.tau_l, wl.tau_h, wl.beta)
+            if self._apool is not None:
+                self.g_slot.add_(1)
+                self.g_slot.remainder_(self.input_pool)
+        self.g_slot.fill_(t % self.input_pool if self._apool is not None else 0)
         self.graph = g
+
+    def _put_small(self, keep):
+        """Upload keep counts and the active sequences' current rewards into g_small."""
+        rw = np.asarray([self.current_reward(s) for s in self.active], np.float32).view(np.int32)
+        self.staging.put(np.concatenate([np.asarray(keep, np.int32), rw]), torch.int32, out=self.g_small.view(-1))
 
     def current_reward(self, s: int) -> float:
         return float(self.hist[s][-1]) if self.hist[s] else 0.0
@@ -329,10 +348,8 @@ class Trace:
         wl = self.wl
         if self.use_graph:
             if self.graph is None:
-                self._capture()
-            if self._apool is not None:
-                self.g_in.copy_(self._apool[t % self.input_pool])
-            else:
+                self._capture(t)
+            if self._apool is None:
                 q, kn, vn = self.active_inputs(t)
                 self.g_q.copy_(q)
                 self.g_kn.copy_(kn)
@@ -398,7 +415,11 @@ class Trace:
             q_win = None
             if info:
                 q_win = self.active_window_queries(t)
-                keep_dev = self.staging.put(keep, torch.int32)
+                if self.use_graph and self.graph is not None:
+                    self._put_small(keep)  # keep counts and the new rewards together
+                    keep_dev = self.g_small[0]
+                else:
+                    keep_dev = self.staging.put(keep, torch.int32)
                 # only the sequences compressed now are scored (keep == L skips the rest)
                 reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
                                       self.ws_score, keep=keep_dev)
@@ -424,6 +445,6 @@ class Trace:
             ev.boundaries.append((t, info, sorted(gone)))
             if gone:
                 self._drop(gone)
-            elif self.use_graph and self.graph is not None:
-                self.staging.put([self.current_reward(s) for s in self.active], torch.float32, out=self.g_rw)
+            elif self.use_graph and self.graph is not None and not info:
+                self._put_small(keep)  # the new rewards (the keep row is not read)
         return ev
