@@ -2,10 +2,9 @@
 // attention whose cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2).
 //
 // bf16 path (decode_tma): a persistent split-K flash-decode, one CTA of 8 warps per
-// SM.  Every CTA first builds the same work plan from lens: a key-chunk length C
-// chosen so the total number of (unit, chunk) items is several per warp, and the
-// prefix sum of chunks per unit.  Each warp's first two items are dealt out
-// statically, round-robin over the CTAs; the rest come from an atomic counter.
+// SM.  Every CTA first builds the same work plan from lens: the prefix sum of 16-key
+// blocks per unit, with the blocks of all units laid end to end and cut into one equal
+// contiguous range per warp (a stream-K split: balanced to one block, no work queue).
 // An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
 // (128-byte swizzled 16 x 64 tiles of K and V) into the warp's 3-stage ring and the
 // warp waits on the stage's mbarrier (bounded).  QK^T and PV run on mma.sync
@@ -213,11 +212,11 @@ __device__ __forceinline__ uint32_t word(const uint4 &v, int x)
 
 constexpr int kDecodeWarps = 8;       // warps per CTA (one CTA per SM)
 constexpr int kDecodeStages = 3;      // ring stages per warp
-constexpr int kItemsPerWarp = 4;      // target work items per warp (fewer, larger items pay less per-item cost)
-constexpr int kMaxTmaUnits = 3072;    // two plan entries per unit kept in shared memory
+constexpr int kMaxTmaUnits = 8192;    // one plan entry per unit kept in shared memory
 constexpr long long kSpinLimit = 1LL << 24;  // bounded mbarrier waits (about a second)
 constexpr float kLazyLog2 = 8.f;             // output rescale threshold (log2 units)
-constexpr int kDecodeMinChunk = 256;         // shortest full chunk (keys): a split costs a merge
+constexpr int kMinBlocksPerWarp = 4;         // fewer working warps rather than shorter ranges
+constexpr int kMaxWholeBlocks = 16;          // units of at most this many blocks are never cut
 
 template <int D> struct TmaLayout {
     static constexpr int HALVES = D / 64;             // 128-byte boxes per row
@@ -226,10 +225,14 @@ template <int D> struct TmaLayout {
     static constexpr int RING = kDecodeWarps * kDecodeStages * STAGE;
 };
 
+// the largest plan fits beside the d = 128 ring (227 KB per CTA, about 1 KB of it static)
+static_assert(1024 + TmaLayout<128>::RING + (kMaxTmaUnits + 1) * 4 + 1024 <= 227 * 1024, "decode smem budget");
+static_assert(kMaxTmaUnits * 4 <= TmaLayout<64>::RING, "lengths are staged in the ring");
+
 template <int D>
 size_t tma_smem_bytes(int units)
 {
-    return 1024 + (size_t)TmaLayout<D>::RING + 2 * (size_t)(units + 1) * sizeof(int);
+    return 1024 + (size_t)TmaLayout<D>::RING + (size_t)(units + 1) * sizeof(int);
 }
 
 // Byte offset of 16-byte chunk ch (0..7) of row rr inside a 128B-swizzled 16-row box.
@@ -245,11 +248,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     constexpr int MT = D / 16;  // m-tiles of PV (d on M)
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NW][S];
-    __shared__ long long sm_red[NW];
-    __shared__ int sm_scan[NW], sm_scan2[NW];
+    __shared__ int sm_scan[NW];
     const uint32_t raw0 = (uint32_t)__cvta_generic_to_shared(smem_raw);
     const uint32_t ring0 = (raw0 + 1023u) & ~1023u;
-    int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // 2 x [units + 1]
+    int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
     const uint32_t my_ring = ring0 + (uint32_t)wid * S * STAGE;
@@ -265,11 +267,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     __syncwarp();
 
     // ---- plan: identical in every CTA (lens are not modified until every warp is done).
-    // Unit u splits into nf_u = le_u / C full chunks and, when le_u % C != 0 (or the unit
-    // is empty), one shorter tail chunk.  Items are handed out full chunks first, tails
-    // last, so the final items are short and the end of the launch drains evenly.
-    int *pre_f = sm_pre;              // [units + 1] prefix of full chunks
-    int *pre_t = sm_pre + units + 1;  // [units + 1] prefix of tail chunks
+    // Each unit's keys form nb_u = ceil(le_u / 16) blocks; the blocks of all units are laid
+    // end to end (prefix pb) and every working warp takes one contiguous range of equal
+    // length, cut across unit boundaries (a stream-K split).  A unit cut between warps
+    // leaves partial (max, sum, output) triples that its last piece merges.  Short units
+    // (<= kMaxWholeBlocks blocks) are never cut: a range start inside one moves back to
+    // the unit's start, since there a merge costs more than the imbalance it removes.
+    int *pb = sm_pre;  // [units + 1] prefix of blocks
     const int seg = (units + blockDim.x - 1) / blockDim.x;
     const int u_lo = min(units, tid * seg), u_hi = min(units, u_lo + seg);
     auto eff_len = [&](int u) {
@@ -298,67 +302,41 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
     }
     __syncthreads();
-    long long tot = 0;
-    for (int u = u_lo; u < u_hi; ++u) tot += len_sm[u];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
-    if (lane == 0) sm_red[wid] = tot;
-    __syncthreads();
-    tot = 0;
-    for (int w2 = 0; w2 < NW; ++w2) tot += sm_red[w2];
-    const int total_warps = gridDim.x * NW;
-    const long long target = min((long long)kDecodeMaxTarget, (long long)kItemsPerWarp * total_warps);
-    long long Cl = (tot + target - 1) / target;
-    Cl = ((Cl + 63) / 64) * 64;
-    if (Cl < kDecodeMinChunk) Cl = kDecodeMinChunk;
-    const int C = (int)Cl;
-    int my_f = 0, my_t = 0;
-    for (int u = u_lo; u < u_hi; ++u) {
-        const int le = len_sm[u];
-        my_f += le / C;
-        my_t += (le % C != 0 || le == 0) ? 1 : 0;
-    }
     {
-        int f = my_f, t2 = my_t;
+        int my_b = 0;
+        for (int u = u_lo; u < u_hi; ++u) my_b += (len_sm[u] + 15) >> 4;
+        int f = my_b;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int nf = __shfl_up_sync(0xffffffffu, f, o), nt = __shfl_up_sync(0xffffffffu, t2, o);
-            if (lane >= o) {
-                f += nf;
-                t2 += nt;
-            }
+            const int nf = __shfl_up_sync(0xffffffffu, f, o);
+            if (lane >= o) f += nf;
         }
-        if (lane == 31) {
-            sm_scan[wid] = f;
-            sm_scan2[wid] = t2;
-        }
+        if (lane == 31) sm_scan[wid] = f;
         __syncthreads();
-        int rf = f - my_f, rt = t2 - my_t;
-        for (int w2 = 0; w2 < wid; ++w2) {
-            rf += sm_scan[w2];
-            rt += sm_scan2[w2];
-        }
+        int rb = f - my_b;
+        for (int w2 = 0; w2 < wid; ++w2) rb += sm_scan[w2];
         for (int u = u_lo; u < u_hi; ++u) {
-            pre_f[u] = rf;
-            pre_t[u] = rt;
-            const int le = len_sm[u];
-            rf += le / C;
-            rt += (le % C != 0 || le == 0) ? 1 : 0;
+            pb[u] = rb;
+            rb += (len_sm[u] + 15) >> 4;
         }
-        if (tid == blockDim.x - 1) {
-            pre_f[units] = rf;
-            pre_t[units] = rt;
-        }
+        if (tid == blockDim.x - 1) pb[units] = rb;
     }
     __syncthreads();
-    const int NF = pre_f[units];
-    const int total_items = NF + pre_t[units];
+    const int NB = pb[units];
+    const int total_warps = gridDim.x * NW;
+    // working warps: every one gets at least kMinBlocksPerWarp blocks (or all warps work)
+    const int W = max(1, min(total_warps, NB / kMinBlocksPerWarp));
     const int g = lane >> 2, c = lane & 3;
     const bool out_bf16 = a.out_bf16 != 0;
+    auto wstart = [&](int w) { return (int)((long long)w * NB / W); };  // ideal first block of warp w
+    auto owner = [&](int b) { return (int)(((long long)(b + 1) * W - 1) / NB); };  // ideal owner of block b
 
-    // dispatch index -> (unit, chunk) and the chunk's key range
+    // A piece: the part of unit u inside one warp's block range.  A unit cut between warps
+    // wf .. wf+nsplit-1 keeps warp w's partial in slot 2w (the warp's first piece) or 2w+1
+    // (its last piece): only those two pieces of a warp can be partial.  Only long units
+    // are cut, and no range start moves inside a long unit, so there the ideal owners hold.
     struct Item {
-        int u, split, first, nsplit, le, k0, k1, Lapp, nblk;
+        int u, ub, wf, nsplit, slot, slot0, le, k0, k1, Lapp, nblk;
     };
     auto last_le = [](const int *pre, int units_, int d) {  // largest u with pre[u] <= d
         int lo = 0, hi = units_ - 1;
@@ -368,39 +346,66 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         return lo;
     };
-    auto meta = [&](int d) {
+    auto snap = [&](int b) {  // a range start inside a short unit moves to the unit's start
+        if (b >= NB) return NB;
+        const int u = last_le(pb, units, b);
+        return pb[u + 1] - pb[u] <= kMaxWholeBlocks ? pb[u] : b;
+    };
+    // static deal interleaved across CTAs (warp wid of every CTA before warp wid+1 of
+    // any): with fewer working warps than warps the work still spreads over all SMs
+    const int gw = wid * (int)gridDim.x + (int)blockIdx.x;
+    const bool working = gw < W;
+    const int b_end = working ? snap(wstart(gw + 1)) : 0;
+    int b_next = working ? snap(wstart(gw)) : 0;
+    int eu = gw;  // next unit this warp checks for emptiness (empty units: no blocks)
+    auto next_item = [&]() {
         Item it;
         it.nblk = -1;  // no item
-        if (d >= total_items) return it;
-        int u, split;
-        if (d < NF) {
-            u = last_le(pre_f, units, d);
-            split = d - pre_f[u];
-        } else {
-            u = last_le(pre_t, units, d - NF);
-            split = pre_f[u + 1] - pre_f[u];
+        if (b_next < b_end) {
+            const int u = last_le(pb, units, b_next);  // the nonempty unit holding block b_next
+            const int ub = pb[u], ue = pb[u + 1];
+            const int bend = min(b_end, ue);
+            const int le_raw = eff_len(u);
+            it.u = u;
+            it.ub = ub;
+            it.le = le_raw >= 0 ? le_raw : 0;
+            it.Lapp = (le_raw >= 0 && a.append) ? it.le - 1 : -1;
+            it.k0 = (b_next - ub) * 16;
+            it.k1 = min((bend - ub) * 16, it.le);
+            it.nblk = bend - b_next;
+            if (ue - ub <= kMaxWholeBlocks) {  // a short unit: always whole
+                it.wf = gw;
+                it.nsplit = 1;
+                it.slot = it.slot0 = 0;
+            } else {
+                it.wf = owner(ub);
+                it.nsplit = owner(ue - 1) - it.wf + 1;
+                it.slot0 = 2 * it.wf + (snap(wstart(it.wf)) < ub ? 1 : 0);  // warp wf's slot
+                it.slot = gw == it.wf ? it.slot0 : 2 * gw;
+            }
+            b_next = bend;
+            return it;
         }
-        const int le_raw = eff_len(u);
-        it.u = u;
-        it.split = split;
-        it.first = pre_f[u] + pre_t[u];
-        it.nsplit = (pre_f[u + 1] - pre_f[u]) + (pre_t[u + 1] - pre_t[u]);
-        it.le = le_raw >= 0 ? le_raw : 0;
-        it.Lapp = (le_raw >= 0 && a.append) ? it.le - 1 : -1;
-        it.k0 = min(split * C, it.le);
-        it.k1 = min(it.k0 + C, it.le);
-        it.nblk = (it.k1 - it.k0 + 15) / 16;
+        while (eu < units) {  // units without keys: zero output, lse = -inf
+            const int u = eu;
+            eu += total_warps;
+            if (pb[u + 1] == pb[u]) {
+                const int le_raw = eff_len(u);
+                it.u = u;
+                it.ub = pb[u];
+                it.le = 0;
+                it.Lapp = -1;
+                it.k0 = it.k1 = 0;
+                it.nblk = 0;
+                it.wf = 0;
+                it.nsplit = 1;
+                it.slot = it.slot0 = 0;
+                (void)le_raw;
+                return it;
+            }
+        }
         return it;
     };
-    // Items 0 .. 2*total_warps-1 are dealt out statically (two per warp);
-    // the counter hands out the rest.  A warp takes its counter ticket one item ahead
-    // (issued when an item starts, read when it ends) so the atomic's latency is hidden.
-    auto ticket = [&]() {
-        int d = 0;
-        if (lane == 0) d = atomicAdd(&a.counters[0], 1);
-        return d;
-    };
-    auto redeem = [&](int d) { return meta(2 * total_warps + __shfl_sync(0xffffffffu, d, 0)); };
 
     // Q fragments of an item (rows g < G), head dim permuted to match the K chunks:
     // k-step j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
@@ -426,15 +431,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // item into the next one (grabbed one item ahead) so no refill bubble opens between
     // items; the warp consumes blocks in issue order.
     uint32_t issued = 0, consumed = 0;
-    // static deal interleaved across CTAs (warp wid of every CTA before warp wid+1 of
-    // any): a partial round then spreads evenly over the SMs, whose warps share one
-    // TMA unit and one L2 port
-    const int gw = wid * (int)gridDim.x + (int)blockIdx.x;
-    Item cur = meta(gw);
+    Item cur = next_item();
     uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
     if (cur.nblk >= 0) load_q(cur, qa_n);
-    Item nxt = cur.nblk >= 0 ? meta(gw + total_warps) : cur;
-    int tk = 0;  // counter ticket for the item after nxt
+    Item nxt = cur.nblk >= 0 ? next_item() : cur;
     Item pit = cur;  // item the producer is issuing from
     int pblk = 0;
     bool p_on_next = false;
@@ -469,7 +469,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 
     while (cur.nblk >= 0) {
         const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
-        const int first = cur.first, nsplit = cur.nsplit, item = first + cur.split;  // partial slot
+        const int nsplit = cur.nsplit, item = cur.slot, wf = cur.wf, slot0 = cur.slot0;  // partial slots
         const long lb = u / a.Hkv;
         const int h = u % a.Hkv;
         const int G = a.G;
@@ -487,10 +487,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             qa[j][0] = qa_n[j][0];
             qa[j][1] = qa_n[j][1];
         }
-        if (nxt.nblk >= 0) {
-            load_q(nxt, qa_n);  // the next item's queries load while this one streams
-            tk = ticket();
-        }
+        if (nxt.nblk >= 0) load_q(nxt, qa_n);  // the next item's queries load while this one streams
         float o[MT][4];
 #pragma unroll
         for (int t = 0; t < MT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
@@ -676,7 +673,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                     if (s2 < nsplit) {
 #pragma unroll
                         for (int qq = 0; qq < 8; ++qq)
-                            if (qq < G) Mq[qq] = fmaxf(Mq[qq], __ldcg(a.part_ml + ((size_t)(first + s2) * G + qq) * 2));
+                            if (qq < G)
+                                Mq[qq] = fmaxf(Mq[qq], __ldcg(a.part_ml + ((size_t)(s2 ? 2 * (wf + s2) : slot0) * G + qq) * 2));
                     }
                 }
 #pragma unroll
@@ -693,7 +691,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 }
 #pragma unroll 2
                 for (int s2 = 0; s2 < nsplit; ++s2) {
-                    const size_t it0 = (size_t)(first + s2) * G;
+                    const size_t it0 = (size_t)(s2 ? 2 * (wf + s2) : slot0) * G;
 #pragma unroll
                     for (int qq = 0; qq < 8; ++qq) {
                         if (qq < G && Mq[qq] != -INFINITY) {
@@ -730,7 +728,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         // advance: the producer may already be streaming the next item's blocks
         cur = nxt;
-        nxt = cur.nblk >= 0 ? redeem(tk) : cur;
+        nxt = cur.nblk >= 0 ? next_item() : cur;
         if (p_on_next) {
             p_on_next = false;
         } else {
@@ -799,7 +797,9 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.c2 = scale * kLog2e;
     a.err = err;
     const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
-    if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31)) {
+    // partial slots: two per warp of the grid
+    const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.max_items;
+    if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31) && slots_fit) {
         CUtensorMap mk, mv;
         if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {
             cudaError_t e = cudaMemsetAsync(ws.counters, 0, (size_t)(2 + a.units) * 4, s);
