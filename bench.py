@@ -458,8 +458,8 @@ def run_trace(args):
                                f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
                                f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
                    "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically",
-                   "per_token_launch": "captured CUDA graph (decode + penalty)" if use_graph
-                   else "direct calls"},
+                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty)"
+                   if use_graph else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),
                   "stops": sum(1 for p in ev.probes if p[2]),
