@@ -15,6 +15,7 @@ Each wrapper names the paper passage it follows:
   gather_unit                   -- compaction to m rows, Sec. 3.2
   decode_unit / decode_batch    -- softmax attention over the compacted cache
   penalty_band / reflect_penalty-- Eq. 3 and Eq. 4, Sec. 3.3
+  penalty_sample                -- Eq. 3-4, then a draw from softmax(z~) (Sec. 3.3)
   probe_trigger                 -- two consecutive top-band rewards, Sec. 3.3
   answer_ppl                    -- Eq. 5 and Eq. 6, Sec. 3.3
 """
@@ -89,6 +90,9 @@ def _bind(lib):
     lib.oracle_reflect_penalty.argtypes = [_f32p, c_int, c_int, _i32p, c_int, _f32p, c_float,
                                            c_float, c_float, ctypes.c_void_p]
     lib.oracle_reflect_penalty.restype = c_int
+    lib.oracle_penalty_sample.argtypes = [_f32p, c_int, c_int, _i32p, c_int, _f32p, c_float, c_float, c_float,
+                                          _f32p, _i32p, _f64p, _f64p]
+    lib.oracle_penalty_sample.restype = c_int
     lib.oracle_probe_trigger.argtypes = [c_float, c_float, c_float]
     lib.oracle_probe_trigger.restype = c_int
     lib.oracle_answer_ppl.argtypes = [_f32p, _i32p, ctypes.c_void_p, c_int, c_int, c_int, c_float,
@@ -208,6 +212,20 @@ def reflect_penalty(logits, ids, rewards, tau_l=0.4, tau_h=0.8, beta=4.0):
     bad = _load().oracle_reflect_penalty(z, B, V, ids, int(ids.size), r, float(tau_l), float(tau_h),
                                          float(beta), beta_out.ctypes.data)
     return z, beta_out, int(bad)
+
+
+def penalty_sample(logits, ids, rewards, uniforms, tau_l=0.4, tau_h=0.8, beta=4.0):
+    """Eq. 3-4 on a copy of logits [B,V], then one inversion draw per row at uniforms [B].
+    Returns (penalised logits, tokens [B] int32, cdf_lo [B], cdf_hi [B], #ignored ids)."""
+    z = _f32(logits).copy()
+    B, V = z.shape
+    ids = _i32(ids).ravel()
+    tok = np.zeros(B, np.int32)
+    lo = np.zeros(B, np.float64)
+    hi = np.zeros(B, np.float64)
+    bad = _load().oracle_penalty_sample(z, B, V, ids, int(ids.size), _f32(rewards).ravel(), float(tau_l),
+                                        float(tau_h), float(beta), _f32(uniforms).ravel(), tok, lo, hi)
+    return z, tok, lo, hi, int(bad)
 
 
 def probe_trigger(v_prev: float, v_cur: float, tau_h: float = 0.8) -> bool:

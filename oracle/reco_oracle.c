@@ -29,6 +29,8 @@
  *     float32 scores (the precision the kernel decides in).
  *   - Eq. 3 bands compare float32 rewards with float32 thresholds.
  *   - Eq. 4 subtracts the band penalty once per distinct id of R.
+ *   - Sampling after Eq. 4: temperature 1, one draw per row by inversion of the
+ *     CDF in token-index order at a uniform draw the caller supplies.
  *   - Eq. 5 uses raw logits, natural log; an empty answer has PPL = NaN, no stop.
  *   - Early-stop probe: v_{i-1} >= tau_h and v_i >= tau_h.
  */
@@ -280,6 +282,64 @@ int oracle_reflect_penalty(float *logits, int B, int V, const int32_t *ids, int 
             }
     }
     free(in_R);
+    return bad;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Sampling from the penalised logits (Sec. 3.3, after Eq. 4: the next token  */
+/* is drawn from softmax(z~), temperature 1).  Eq. 3 + Eq. 4 are applied in    */
+/* place first (oracle_reflect_penalty), then each row draws one token by      */
+/* inversion: with p = softmax(z~ row) and the given uniform u[b], the token   */
+/* is the smallest j with p_j > 0 and sum_{i<=j} p_i > u.  If rounding leaves  */
+/* no such j (u at the top of [0, 1)), the last j with p_j > 0 is taken; a row */
+/* of -inf logits gets -1.  cdf_lo / cdf_hi (may be NULL) receive             */
+/* sum_{i<j} p_i and sum_{i<=j} p_i of the chosen token.  Returns the number  */
+/* of ids outside [0, V).                                                      */
+/* ------------------------------------------------------------------------- */
+int oracle_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids,
+                          const float *rewards, float tau_l, float tau_h, float beta,
+                          const float *uniforms, int32_t *tokens, double *cdf_lo, double *cdf_hi)
+{
+    int bad = oracle_reflect_penalty(logits, B, V, ids, n_ids, rewards, tau_l, tau_h, beta, NULL);
+    for (int b = 0; b < B; ++b) {
+        const float *z = logits + (size_t)b * V;
+        double M = -INFINITY;
+        for (int j = 0; j < V; ++j)
+            if ((double)z[j] > M) M = (double)z[j];
+        int tok = -1;
+        double lo = 0.0, hi = 0.0;
+        if (M != -INFINITY) {
+            double Z = 0.0;
+            for (int j = 0; j < V; ++j) Z += exp((double)z[j] - M);
+            double u = (double)uniforms[b];
+            double c = 0.0;
+            int last = -1;
+            double last_lo = 0.0;
+            for (int j = 0; j < V; ++j) {
+                double p = exp((double)z[j] - M) / Z;
+                double prev = c;
+                c += p;
+                if (p > 0.0) {
+                    last = j;
+                    last_lo = prev;
+                }
+                if (c > u && p > 0.0) {
+                    tok = j;
+                    lo = prev;
+                    hi = c;
+                    break;
+                }
+            }
+            if (tok < 0) {
+                tok = last;
+                lo = last_lo;
+                hi = c;
+            }
+        }
+        tokens[b] = tok;
+        if (cdf_lo) cdf_lo[b] = lo;
+        if (cdf_hi) cdf_hi[b] = hi;
+    }
     return bad;
 }
 

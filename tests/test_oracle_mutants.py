@@ -65,6 +65,16 @@ MUTANTS = {
     "eq5 sign of the mean log-probability": (
         "ppl[b] = exp(-sum_lp / (double)nv);", "ppl[b] = exp(sum_lp / (double)nv);",
         [P.test_eq5_golden]),
+    "sampling boundary taken inclusive": (
+        "if (c > u && p > 0.0) {", "if (c >= u && p > 0.0) {",
+        [P.test_sample_golden_cdf_boundaries]),
+    "sampling before the penalty": (
+        "int bad = oracle_reflect_penalty(logits, B, V, ids, n_ids, rewards, tau_l, tau_h, beta, NULL);",
+        "int bad = 0;",
+        [P.test_sample_draws_after_the_penalty]),
+    "sampling normaliser without the max shift": (
+        "for (int j = 0; j < V; ++j) Z += exp((double)z[j] - M);", "for (int j = 0; j < V; ++j) Z += exp((double)z[j]);",
+        [P.test_sample_golden_cdf_boundaries]),
     "eq5 log-sum-exp without the max": (
         "sum_lp += (double)z[x] - (M + log(Z));", "sum_lp += (double)z[x] - log(Z);",
         [P.test_eq5_matches_torch_cross_entropy_and_ragged_lengths]),

@@ -371,3 +371,70 @@ def test_eq6_stop_boundary_is_inclusive():
     ppl, stop = oracle.answer_ppl(np.zeros((1, 2, 3), np.float32), np.zeros((1, 2), np.int32),
                                   np.array([0], np.int32))
     assert math.isnan(ppl[0]) and not stop[0]  # empty answer: no perplexity, no stop
+
+
+# ---------------------------------------------------------------- sampling after Eq. 4 --------
+def _sample(z, u, ids=(), rewards=None, **kw):
+    z = np.atleast_2d(np.asarray(z, np.float32))
+    B = z.shape[0]
+    rewards = np.zeros(B, np.float32) if rewards is None else rewards
+    return oracle.penalty_sample(z, np.asarray(ids, np.int32), rewards, np.asarray(u, np.float32), **kw)
+
+
+def test_sample_golden_cdf_boundaries():
+    g = gold("sample_inversion.json")
+    t = g["two_token"]
+    for u, tok in t["cases"]:
+        assert _sample([t["logits"]], [u])[1][0] == tok, (u, tok)
+    un = g["uniform"]
+    for u, tok in un["cases"]:
+        assert _sample(np.zeros((1, un["V"])), [u])[1][0] == tok, (u, tok)
+    oh = g["one_hot"]
+    z = np.zeros((1, oh["V"]), np.float32)
+    z[0, oh["hot"]] = oh["boost"]
+    for u in oh["uniforms"]:
+        assert _sample(z, [u])[1][0] == oh["hot"]
+    m = g["masked"]
+    zm = [float(x) for x in m["logits"]]
+    for u, tok in m["cases"]:
+        assert _sample([zm], [u])[1][0] == tok, (u, tok)
+
+
+def test_sample_draws_after_the_penalty():
+    g = gold("sample_inversion.json")["penalty"]
+    for c in g["cases"]:
+        _, tok, _, _, _ = _sample([g["z"]], [c["u"]], g["ids"], np.array([c["v"]], np.float32),
+                                  tau_l=g["tau_l"], tau_h=g["tau_h"], beta=g["beta"])
+        assert tok[0] == c["token"], c
+
+
+def test_sample_matches_searchsorted_on_the_cumulative_softmax():
+    rng = np.random.default_rng(21)
+    B, V = 64, 300
+    z = (rng.standard_normal((B, V)) * 2).astype(np.float32)
+    ids = rng.choice(V, 10, replace=False).astype(np.int32)
+    rw = rng.uniform(0, 1, B).astype(np.float32)
+    u = rng.uniform(0, 1, B).astype(np.float32)
+    zp, tok, lo, hi, bad = _sample(z, u, ids, rw)
+    assert bad == 0
+    for b in range(B):
+        p = scipy.special.softmax(zp[b].astype(np.float64))
+        cdf = np.cumsum(p)
+        ref = int(np.searchsorted(cdf, float(u[b]), side="right"))
+        if abs(cdf[ref] - u[b]) > 1e-12 and (ref == 0 or abs(cdf[ref - 1] - u[b]) > 1e-12):
+            assert tok[b] == ref, (b, tok[b], ref)
+        assert abs(lo[b] - (cdf[tok[b] - 1] if tok[b] else 0.0)) < 1e-12 and abs(hi[b] - cdf[tok[b]]) < 1e-12
+
+
+def test_sample_stratified_counts_follow_the_probabilities():
+    """With stratified draws u_k = (k + 1/2)/N, inversion gives token j exactly the number of
+    grid points inside its CDF interval, i.e. N p_j to within one, for every j."""
+    rng = np.random.default_rng(22)
+    V, N = 50, 4000
+    z = (rng.standard_normal(V) * 2).astype(np.float32)
+    u = ((np.arange(N) + 0.5) / N).astype(np.float32)
+    _, tok, _, _, _ = _sample(np.repeat(z[None], N, 0), u)
+    counts = np.bincount(tok, minlength=V)
+    p = scipy.special.softmax(z.astype(np.float64))
+    assert np.abs(counts - N * p).max() <= 1.0 + 1e-6, np.abs(counts - N * p).max()
+    assert counts.sum() == N
