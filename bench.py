@@ -268,6 +268,43 @@ def workload_name(wl):
 
 
 # ------------------------------------------------------------------ GPU arm
+def time_penalty_sample(wl, dev, n_buf=32, reps=4):
+    """The penalty followed by one draw per sequence (reco_penalty_sample) on the workload's
+    vocabulary, timed apart from the step: n_buf logits buffers (more bytes than L2) are
+    visited in turn so every launch reads its logits from HBM.  Algorithmic bytes per launch:
+    the logits once, plus one segment per row read again and the penalised ids written."""
+    from paper_2608_04771_gb300 import reco
+    from paper_2608_04771_gb300 import workloads as W
+    zs = [W.make_vocab_logits(wl, dev, stream=60 + i) for i in range(n_buf)]
+    ids = torch.from_numpy(W.make_reflection_ids(wl)).to(dev)
+    rw = torch.from_numpy(W.make_reward_history(wl)[:, -1].copy()).to(dev)
+    u = torch.from_numpy(W.make_draws(wl, wl.batch)).to(dev)
+    tok = torch.empty(wl.batch, dtype=torch.int32, device=dev)
+    ws = reco.sample_workspace(wl.batch, wl.vocab, dev)
+    for z in zs[:4]:
+        reco.reco_penalty_sample(z, ids, rw, u, tok, ws, wl.tau_l, wl.tau_h, wl.beta)
+    torch.cuda.synchronize()
+    # the n_buf calls as one CUDA graph, so the launches are not paced by the host
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="relaxed"):
+        for z in zs:
+            reco.reco_penalty_sample(z, ids, rw, u, tok, ws, wl.tau_l, wl.tau_h, wl.beta)
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        g.replay()
+    b.record()
+    b.synchronize()
+    reco.reco_check()
+    ms = a.elapsed_time(b) / (reps * n_buf)
+    byts = 4.0 * wl.batch * wl.vocab + 4.0 * wl.batch * min(wl.vocab, 4096) + 8.0 * wl.batch * wl.n_ids
+    return {"ms_per_launch": ms, "GB/s": byts / ms / 1e6, "rows": wl.batch, "vocab": wl.vocab,
+            "timing": f"{n_buf} logits buffers visited in turn ({n_buf * 4 * wl.batch * wl.vocab / 1e6:.0f} MB > L2) "
+                      "by one captured graph, outside the timed step"}
+
+
 def run_gpu(args, wl):
     from paper_2608_04771_gb300 import build as B
     from paper_2608_04771_gb300 import driver, reco
@@ -347,6 +384,7 @@ def run_gpu(args, wl):
         kernels["penalty"] = {"ms_per_launch": pen_ms}
         kernels["ppl"] = {"ms": statistics.mean(ph["ppl"]),
                           "GB/s": alg["ppl_bytes"] / statistics.mean(ph["ppl"]) / 1e6}
+        kernels["penalty_sample"] = time_penalty_sample(wl, dev)
 
     e2e = run_e2e(hp, wl, args, world) if not args.no_e2e else None
     clocks = clk.summary()
@@ -450,7 +488,7 @@ def run_trace(args):
     row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes
     full_peak = spec.batch * (spec.prompt + spec.generated) * row_bytes
     line = {
-        "metric": "step-loop trace: generated tokens/s (decode + penalty every token, compression at step "
+        "metric": "step-loop trace: generated tokens/s (decode + penalty + draw every token, compression at step "
                   "boundaries, answer probes), 1xGB300",
         "value": ev.generated / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1, "ms_total": ms, "wall_s": wall,
         "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
@@ -458,7 +496,7 @@ def run_trace(args):
                                f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
                                f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
                    "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically",
-                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty)"
+                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty and draw)"
                    if use_graph else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),

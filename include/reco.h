@@ -61,7 +61,13 @@ typedef struct {
     reco_dtype dtype; /* RECO_F32 or RECO_BF16 */
 } reco_kv;
 
-typedef enum { RECO_OP_SCORE = 0, RECO_OP_SELECT = 1, RECO_OP_DECODE = 2, RECO_OP_PPL = 3 } reco_op;
+typedef enum {
+    RECO_OP_SCORE = 0,
+    RECO_OP_SELECT = 1,
+    RECO_OP_DECODE = 2,
+    RECO_OP_PPL = 3,
+    RECO_OP_SAMPLE = 4
+} reco_op;
 
 /* ---------------------------------------------------------------- host helpers */
 
@@ -84,8 +90,10 @@ int reco_penalty_band(float v, float tau_l, float tau_h);
 int reco_probe_trigger(float v_prev, float v_cur, float tau_h);
 
 /* Workspace bytes the device call `op` needs for this cache shape (and window w
- * for RECO_OP_SCORE, answer batch B*n passed in `w` for RECO_OP_PPL).  The size
- * does not depend on the device or on lens.  Alignment: 256 bytes.            */
+ * for RECO_OP_SCORE, answer batch B*n passed in `w` for RECO_OP_PPL).  For
+ * RECO_OP_SAMPLE, kv is NULL, `w` is the vocabulary size V and the result is the
+ * size per sequence (reco_penalty_sample needs B times it).  The size does not
+ * depend on the device or on lens.  Alignment: 256 bytes.                      */
 reco_status reco_workspace_bytes(reco_op op, const reco_kv *kv, int w, size_t *bytes_out);
 
 /* Thread-local message describing the last non-OK status ("" if none).        */
@@ -168,6 +176,26 @@ reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new
 reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
                                  const float *rewards, float tau_l, float tau_h, float beta,
                                  float *beta_out, cudaStream_t stream);
+
+/* Eq. 3 + Eq. 4 in place, then one draw per sequence from softmax of the penalised
+ * logits (Sec. 3.3: while the next step is generated its tokens are sampled from
+ * softmax of the penalised logits, temperature 1), by inversion of the distribution
+ * in token order at a draw the caller supplies:
+ *   p         = softmax(logits[b, :]) after the penalty,
+ *   tokens[b] = the smallest j with p_j > 0 and sum_{i<=j} p_i > uniforms[b];
+ * if rounding leaves no such j (a draw at the top of [0, 1), or NaN), the last j with
+ * p_j > 0; a row whose logits are all -inf gets -1.  Logits must be finite or -inf.
+ *   logits, ids, n_ids, rewards, tau_l, tau_h, beta, beta_out : as reco_reflect_penalty
+ *            (the logits are penalised in place exactly as reco_reflect_penalty does)
+ *   uniforms : [B] float32 (device), one draw in [0, 1) per sequence
+ *   tokens   : [B] int32 (device, written)
+ *   ws       : at least B * reco_workspace_bytes(RECO_OP_SAMPLE, NULL, V) bytes
+ * V may be at most 4194304.  The probabilities are float32 (2^x on the special-
+ * function unit), so a draw within about 1e-5 of a boundary of the cumulative
+ * distribution may select the neighbouring token.                              */
+reco_status reco_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
+                                float tau_l, float tau_h, float beta, const float *uniforms, int32_t *tokens,
+                                float *beta_out, void *ws, size_t ws_bytes, cudaStream_t stream);
 
 /* Eq. 5 + Eq. 6 (Sec. 3.3, early stopping via answer confidence):
  *   lp[b,t] = logits[b,t,tokens[b,t]] - logsumexp(logits[b,t,:])   (natural log)

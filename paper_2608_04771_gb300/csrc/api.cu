@@ -194,6 +194,11 @@ reco_status reco_workspace_bytes(reco_op op, const reco_kv *kv, int w, size_t *b
         if ((st = check_kv(kv, false)) != RECO_OK) return st;
         *bytes_out = reco::decode_ws_layout(*kv, nullptr).bytes;
         return RECO_OK;
+    case RECO_OP_SAMPLE:
+        if (w < 1 || w > reco::kSampleSeg * reco::kSampleMaxSeg)
+            return fail(RECO_EINVAL, "vocabulary size %d outside [1, %d]", w, reco::kSampleSeg * reco::kSampleMaxSeg);
+        *bytes_out = (size_t)((w + reco::kSampleSeg - 1) / reco::kSampleSeg) * 8;
+        return RECO_OK;
     case RECO_OP_PPL:
         if (w < 0) return fail(RECO_EINVAL, "answer rows B*n must be >= 0");
         *bytes_out = reco::align256((size_t)w * 4);
@@ -300,6 +305,30 @@ reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids
     if (st != RECO_OK) return st;
     cudaError_t e = reco::launch_penalty(logits, B, V, ids, n_ids, rewards, tau_l, tau_h, beta, beta_out, err, stream);
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_reflect_penalty launch");
+}
+
+reco_status reco_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
+                                float tau_l, float tau_h, float beta, const float *uniforms, int32_t *tokens,
+                                float *beta_out, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    if (B < 1 || V < 1 || n_ids < 0) return fail(RECO_EINVAL, "need B >= 1, V >= 1, n_ids >= 0");
+    if (!logits || !rewards || !uniforms || !tokens || (n_ids > 0 && !ids))
+        return fail(RECO_EINVAL, "NULL logits, rewards, uniforms, tokens or ids");
+    if (((uintptr_t)logits | (uintptr_t)rewards | (uintptr_t)uniforms | (uintptr_t)tokens) & 3u)
+        return fail(RECO_EINVAL, "logits, rewards, uniforms and tokens must be 4-byte aligned");
+    if (B > 65535) return fail(RECO_EUNSUPPORTED, "B = %d exceeds 65535", B);
+    if (V > reco::kSampleSeg * reco::kSampleMaxSeg)
+        return fail(RECO_EUNSUPPORTED, "V = %d exceeds %d", V, reco::kSampleSeg * reco::kSampleMaxSeg);
+    if (!(beta >= 0.f)) return fail(RECO_EINVAL, "beta must be >= 0");
+    const size_t nseg = (size_t)(V + reco::kSampleSeg - 1) / reco::kSampleSeg;
+    reco_status st = check_ws(ws, ws_bytes, (size_t)B * nseg * 8);
+    if (st != RECO_OK) return st;
+    if ((uintptr_t)ws & 7u) return fail(RECO_EINVAL, "workspace must be 8-byte aligned");
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_penalty_sample(logits, B, V, ids, n_ids, rewards, tau_l, tau_h, beta, uniforms, tokens,
+                                                beta_out, (float2 *)ws, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_penalty_sample launch");
 }
 
 reco_status reco_answer_ppl(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B, int n, int V,

@@ -12,6 +12,9 @@ namespace reco {
 constexpr int kScoreChunk = 2048;
 // Upper bound on decode split-K work items beyond one per unit.
 constexpr int kDecodeMaxTarget = 16384;
+// Sampling: logits per pass-1 segment, and the most segments a row may have.
+constexpr int kSampleSeg = 4096;
+constexpr int kSampleMaxSeg = 1024;
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -70,6 +73,9 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
 cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
                            const float *rewards, float tau_l, float tau_h, float beta, float *beta_out,
                            unsigned *err, cudaStream_t s);
+cudaError_t launch_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
+                                  float tau_l, float tau_h, float beta, const float *uniforms, int32_t *tokens,
+                                  float *beta_out, float2 *part, unsigned *err, cudaStream_t s);
 cudaError_t launch_ppl(const float *logits, const int32_t *tokens, const int32_t *n_valid, int B, int n,
                        int V, float tau_p, float *ppl, uint8_t *stop, float *lp_ws, unsigned *err,
                        cudaStream_t s);

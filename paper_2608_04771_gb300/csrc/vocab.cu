@@ -4,6 +4,9 @@
 // step reward (float32 compares); Eq. 4 subtracts it from the logit of every
 // reflection token, in place.  R is a set: an id listed twice is penalised once.
 //
+// sample_segments + sample_pick: Eq. 3-4 and then one draw per row from softmax of the
+// penalised logits (Sec. 3.3, temperature 1) by inversion at a caller-supplied uniform.
+//
 // ppl_rows + ppl_finish: Eq. 5 log p(x_t) = z[x_t] - logsumexp(z) per answer row
 // (one CTA per row, one streaming pass with an online max/sum), then per sequence
 // PPL = exp(-mean log p) and the Eq. 6 stop flag PPL <= tau_p.
@@ -41,6 +44,225 @@ cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int 
     int nt = n_ids < 32 ? 32 : (n_ids > 256 ? 256 : ((n_ids + 31) / 32) * 32);
     reflect_penalty_kernel<<<B, nt, 0, s>>>(logits, V, ids, n_ids, rewards, tau_l, tau_h, beta, beta_out,
                                             err);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- penalty + sampling
+// Pass 1, one CTA per (row, segment of kSampleSeg logits): the penalty of Eq. 4 on the
+// ids inside the segment (once per distinct id, one correctly rounded float32
+// subtract), then one streaming read of the segment for its log2-domain (max, sum).
+// Tokens at -inf carry no mass.
+template <int NT>
+__global__ void __launch_bounds__(NT) sample_segments(float *__restrict__ logits, int V, int nseg,
+                                                      const int32_t *__restrict__ ids, int n_ids,
+                                                      const float *__restrict__ rewards, float tau_l, float tau_h,
+                                                      float beta, float *__restrict__ beta_out,
+                                                      float2 *__restrict__ part, unsigned *err)
+{
+    constexpr int PER = kSampleSeg / NT;
+    __shared__ float sm_m[NT / 32], sm_s[NT / 32];
+    const int sg = blockIdx.x, b = blockIdx.y;
+    const int lo = sg * kSampleSeg, hi = min(V, lo + kSampleSeg);
+    float *z = logits + (size_t)b * V;
+    const float v = rewards[b];
+    const float bi = (v <= tau_l) ? 0.f : ((v >= tau_h) ? beta : beta * 0.5f);
+    if (sg == 0 && threadIdx.x == 0 && beta_out) beta_out[b] = bi;
+    for (int i = threadIdx.x; i < n_ids; i += NT) {
+        const int id = ids[i];
+        if (id < 0 || id >= V) {
+            if (b == 0 && sg == 0) raise_error(err, ERR_ID);
+            continue;
+        }
+        if (id < lo || id >= hi || bi == 0.f) continue;
+        bool dup = false;
+        for (int k = 0; k < i && !dup; ++k) dup = ids[k] == id;
+        if (!dup) z[id] = __fsub_rn(z[id], bi);
+    }
+    __syncthreads();  // the segment's penalised logits are visible to the whole CTA
+    float y[PER];
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {  // all loads in flight first
+        const int j = lo + k * NT + (int)threadIdx.x;
+        y[k] = j < hi ? z[j] * kLog2e : -INFINITY;
+    }
+#pragma unroll
+    for (int k = 0; k < PER; ++k) m = fmaxf(m, y[k]);
+    float s = 0.f;
+    if (m != -INFINITY) {
+#pragma unroll
+        for (int k = 0; k < PER; ++k) s += fast_exp2(y[k] - m);  // -inf terms add 0
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+        const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+        lse_merge(m, s, m2, s2);
+    }
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0) {
+        sm_m[wid] = m;
+        sm_s[wid] = s;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float M = sm_m[0], S = sm_s[0];
+        for (int w2 = 1; w2 < NT / 32; ++w2) lse_merge(M, S, sm_m[w2], sm_s[w2]);
+        part[(size_t)b * nseg + sg] = make_float2(M, S);
+    }
+}
+
+// Exclusive block scan of one float per thread (NT threads), in thread order.
+template <int NT>
+__device__ __forceinline__ float block_scan_excl(float x, float *sm_w)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    float incl = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) sm_w[wid] = incl;
+    __syncthreads();
+    float base = 0.f;
+    for (int w2 = 0; w2 < wid; ++w2) base += sm_w[w2];
+    __syncthreads();
+    return base + (incl - x);
+}
+
+// The values v[0..R) of every thread form one sequence in thread order (thread t holds
+// indices first + 0 .. first + R-1).  Returns the first index whose running sum exceeds
+// T among positive values, with the running sum before it; -1 if none (T at or above
+// the total, or NaN).  `last` receives the last index with a positive value (-1: none).
+// A thread whose run the block scan says holds the crossing takes its last positive
+// value when its own sequential sum falls a rounding short of T.
+template <int NT, int R>
+__device__ __forceinline__ int find_crossing(const float (&v)[R], int first, float T, float *sm_w, int *sm_i,
+                                             float *sm_f, float &before, int &last)
+{
+    float run = 0.f;
+    int my_last = -1;
+#pragma unroll
+    for (int k = 0; k < R; ++k) {
+        run += v[k];
+        if (v[k] > 0.f) my_last = first + k;
+    }
+    const float excl = block_scan_excl<NT>(run, sm_w);
+    if (threadIdx.x == 0) {
+        sm_i[0] = -1;
+        sm_i[1] = -1;
+        sm_f[0] = 0.f;
+    }
+    __syncthreads();
+    if (run > 0.f && excl <= T && excl + run > T) {  // at most one thread: the prefix only grows
+        float c = excl, prev = excl + run;  // defaults: the crossing lost to rounding
+        int pick = my_last;
+        bool hit = false;
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const float c0 = c;
+            c += v[k];
+            if (!hit && v[k] > 0.f && c > T) {
+                hit = true;
+                pick = first + k;
+                prev = c0;
+            }
+        }
+        sm_i[0] = pick;
+        sm_f[0] = prev;
+    }
+    if (my_last >= 0) atomicMax(&sm_i[1], my_last);
+    __syncthreads();
+    const int idx = sm_i[0];
+    before = sm_f[0];
+    last = sm_i[1];
+    __syncthreads();
+    return idx;
+}
+
+// Pass 2, one CTA per row.  With M the largest segment max, segment k carries the mass
+// W_k = S_k 2^(m_k - M) and the row Z = sum W_k; the draw u selects T = u Z.  The
+// segment where the running mass first exceeds T is read again and its tokens' masses
+// 2^(z log2e - M) locate the token where the running mass first exceeds what is left of
+// T.  No crossing (u at the top of [0, 1) after rounding, or NaN) takes the last token
+// with mass; a row without mass gets -1.
+template <int NT>
+__global__ void __launch_bounds__(NT) sample_pick(const float *__restrict__ logits, int V, int nseg,
+                                                  const float *__restrict__ uniforms,
+                                                  const float2 *__restrict__ part, int32_t *__restrict__ tokens)
+{
+    constexpr int PER = kSampleSeg / NT;
+    constexpr int SR = kSampleMaxSeg / NT;  // segments per thread
+    __shared__ float sm_w[NT / 32];
+    __shared__ float sm_f[1];
+    __shared__ int sm_i[2];
+    const int b = blockIdx.x, tid = threadIdx.x;
+    const float2 *pp = part + (size_t)b * nseg;
+    float2 q[SR];
+    float M = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < SR; ++k) {
+        const int sg = tid * SR + k;
+        q[k] = sg < nseg ? pp[sg] : make_float2(-INFINITY, 0.f);
+        M = fmaxf(M, q[k].x);
+    }
+    M = warp_max(M);
+    if ((tid & 31) == 0) sm_w[tid >> 5] = M;
+    __syncthreads();
+    M = sm_w[0];
+    for (int w2 = 1; w2 < NT / 32; ++w2) M = fmaxf(M, sm_w[w2]);
+    __syncthreads();
+    if (M == -INFINITY) {  // no token has mass
+        if (tid == 0) tokens[b] = -1;
+        return;
+    }
+    float w[SR];
+    float zsum = 0.f;
+#pragma unroll
+    for (int k = 0; k < SR; ++k) {
+        w[k] = q[k].y > 0.f ? q[k].y * fast_exp2(q[k].x - M) : 0.f;
+        zsum += w[k];
+    }
+    zsum = warp_sum(zsum);
+    if ((tid & 31) == 0) sm_w[tid >> 5] = zsum;
+    __syncthreads();
+    float Z = 0.f;
+    for (int w2 = 0; w2 < NT / 32; ++w2) Z += sm_w[w2];
+    __syncthreads();
+    const float u = uniforms[b];
+    const float T = u != u ? u : fmaxf(u, 0.f) * Z;  // a NaN draw finds no crossing
+    float before;
+    int last_seg;
+    int seg = find_crossing<NT, SR>(w, tid * SR, T, sm_w, sm_i, sm_f, before, last_seg);
+    const bool found = seg >= 0;
+    if (!found) seg = last_seg;
+    const float Tr = found ? fmaxf(T - before, 0.f) : INFINITY;  // left of T inside the segment
+    const float *z = logits + (size_t)b * V;
+    const int first = seg * kSampleSeg + tid * PER;
+    float p[PER];
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int j = first + k;
+        const float y = j < V ? z[j] * kLog2e : -INFINITY;
+        p[k] = y == -INFINITY ? 0.f : fast_exp2(y - M);
+    }
+    float before2;
+    int last_tok;
+    const int tok = find_crossing<NT, PER>(p, first, Tr, sm_w, sm_i, sm_f, before2, last_tok);
+    if (tid == 0) tokens[b] = tok >= 0 ? tok : last_tok;
+}
+
+cudaError_t launch_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
+                                  float tau_l, float tau_h, float beta, const float *uniforms, int32_t *tokens,
+                                  float *beta_out, float2 *part, unsigned *err, cudaStream_t s)
+{
+    const int nseg = (V + kSampleSeg - 1) / kSampleSeg;
+    sample_segments<256><<<dim3(nseg, B), 256, 0, s>>>(logits, V, nseg, ids, n_ids, rewards, tau_l, tau_h, beta,
+                                                      beta_out, part, err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    sample_pick<256><<<B, 256, 0, s>>>(logits, V, nseg, uniforms, part, tokens);
     return cudaGetLastError();
 }
 

@@ -16,12 +16,12 @@ _lib = None
 
 RECO_OK, RECO_EINVAL, RECO_EUNSUPPORTED, RECO_ECUDA, RECO_EDEVICE = range(5)
 RECO_F32, RECO_BF16 = 0, 1
-RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL = range(4)
+RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = range(5)
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_answer_ppl",
-           "reco_answer_ppl_static")
+           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
+           "reco_answer_ppl", "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
 
 
@@ -66,11 +66,12 @@ def lib():
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
+    L.reco_penalty_sample.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp]
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
     L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
                  "reco_score_cache", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty",
-                 "reco_answer_ppl", "reco_answer_ppl_static"):
+                 "reco_penalty_sample", "reco_answer_ppl", "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
     _lib = L
     return L
@@ -178,6 +179,20 @@ def reco_reflect_penalty(logits, ids, rewards, tau_l=0.4, tau_h=0.8, beta=4.0, b
     _ok(lib().reco_reflect_penalty(_ptr(logits), B, V, _ptr(ids), ids.numel(), _ptr(rewards),
                                    float(tau_l), float(tau_h), float(beta), _ptr(beta_out),
                                    _stream(stream)))
+
+
+def sample_workspace(B: int, V: int, device="cuda") -> torch.Tensor:
+    """Workspace for reco_penalty_sample over B rows of V logits."""
+    n = B * reco_workspace_bytes(RECO_OP_SAMPLE, None, V)
+    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+
+
+def reco_penalty_sample(logits, ids, rewards, uniforms, tokens, ws, tau_l=0.4, tau_h=0.8, beta=4.0, beta_out=None,
+                        stream=None):
+    B, V = logits.shape
+    _ok(lib().reco_penalty_sample(_ptr(logits), B, V, _ptr(ids), ids.numel(), _ptr(rewards), float(tau_l),
+                                  float(tau_h), float(beta), _ptr(uniforms), _ptr(tokens), _ptr(beta_out), _ptr(ws),
+                                  ws.numel(), _stream(stream)))
 
 
 def reco_answer_ppl(logits, tokens, n_valid, tau_p, ppl, stop, ws, stream=None):

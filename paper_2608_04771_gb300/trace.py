@@ -3,8 +3,10 @@
 Each sequence generates tokens one at a time; its trajectory is split into steps of
 Poisson(mean) + min tokens (Sec. 3.1 splits at newlines; the lengths here are
 synthetic).  Per token, every active sequence decodes one token (append + attention
-over its ragged cache, all layers in one call) and the reflection penalty (Eq. 3-4)
-is applied to that token's logits with the band of the sequence's latest reward.
+over its ragged cache, all layers in one call), the reflection penalty (Eq. 3-4) is
+applied to that token's logits with the band of the sequence's latest reward, and the
+next token is drawn from softmax of the penalised logits (Sec. 3.3) at a seeded
+uniform draw.
 When a sequence completes a step it receives a reward v_i (Sec. 3.1), and
   * if its cache has grown by at least S tokens since its last compression
     (L - L_{i-1} >= S, Sec. 3.2; L_0 = the prompt; S = 0 compresses at every
@@ -162,7 +164,8 @@ class Trace:
             self._pool = (torch.stack([x[0] for x in ins]), torch.stack([x[1] for x in ins]),
                           torch.stack([x[2] for x in ins]),
                           torch.stack([self._token_logits(t) for t in range(input_pool)]) if wl.vocab else None,
-                          torch.stack([self._window_queries(t) for t in range(8)]))
+                          torch.stack([self._window_queries(t) for t in range(8)]),
+                          torch.stack([self._token_draws(t) for t in range(input_pool)]) if wl.vocab else None)
             del ins
             # the answers of every probe the rewards can trigger, drawn before the loop runs
             for sq in range(spec.batch):
@@ -197,6 +200,13 @@ class Trace:
     def token_logits(self, t: int):
         return self._pool[3][t % self.input_pool].clone() if self._pool else self._token_logits(t)
 
+    def _token_draws(self, t: int):
+        return torch.from_numpy(W.make_draws(self.wl, self.wl.batch, 7_000_000 + t)).to(self.device)
+
+    def token_draws(self, t: int):
+        """[B] uniform draws of token t's sampling step, full batch."""
+        return self._pool[5][t % self.input_pool] if self._pool else self._token_draws(t)
+
     def answer(self, t: int, seq: int):
         """Answer logits / tokens of a probe of sequence `seq` at token t (confident on even probes)."""
         got = self._answers.get((t, seq))
@@ -229,6 +239,11 @@ class Trace:
             return self._slot_view(t % self.input_pool, 3).clone()
         return self._sel(self._token_logits(t), 0)
 
+    def active_draws(self, t: int):
+        if self._apool is not None:
+            return self._slot_view(t % self.input_pool, 4)
+        return self._sel(self._token_draws(t), 0)
+
     def active_window_queries(self, t: int):
         if self._apool is not None:
             return self._awin[t % 8]
@@ -244,9 +259,9 @@ class Trace:
             self._awin = None
             return None
         P = self.input_pool
-        Q, KN, VN, Z, WQ = self._pool
+        Q, KN, VN, Z, WQ, U = self._pool
         sel = (lambda x, d: x) if self._full_batch() else (lambda x, d: x.index_select(d, self.idx_dev))
-        parts = [sel(Q, 2), sel(KN, 2), sel(VN, 2)] + ([] if Z is None else [sel(Z, 1)])
+        parts = [sel(Q, 2), sel(KN, 2), sel(VN, 2)] + ([] if Z is None else [sel(Z, 1), sel(U, 1)])
         self._slot_meta, cols, off = [], [], 0
         for x in parts:
             nb = x[0].numel() * x.element_size()
@@ -279,6 +294,8 @@ class Trace:
         self.lens_dev = torch.tensor(self.lens, dtype=torch.int32, device=self.device).view(1, -1, 1).expand(
             wl.layers, -1, wl.h_kv).contiguous()
         self.ws_ppl = reco.workspace(reco.RECO_OP_PPL, None, wl.n_answer, self.device)
+        self.ws_sample = reco.sample_workspace(self.B, wl.vocab, self.device) if wl.vocab else None
+        self.tokens = None  # the last token's draws, [active] int32
         self.graph = None  # buffers and pointers changed: capture again before the next token
 
     def _drop(self, gone):
@@ -300,13 +317,15 @@ class Trace:
         shapes = [((wl.layers, B, wl.h_q, wl.d), wl.torch_dtype), ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype),
                   ((wl.layers, B, wl.h_kv, wl.d), wl.torch_dtype)]
         if self.ids is not None:
-            shapes.append(((B, wl.vocab), torch.float32))
+            shapes += [((B, wl.vocab), torch.float32), ((B,), torch.float32)]
         protos = [torch.empty(sh, dtype=dt, device="meta") for sh, dt in shapes]
         n = sum((x.numel() * x.element_size() + 255) // 256 * 256 for x in protos)
         self.g_in = torch.zeros(n, dtype=torch.uint8, device=dev)  # q | k_new | v_new | logits
         _, views = _pack(protos, out=self.g_in)
         self.g_q, self.g_kn, self.g_vn = views[:3]
         self.g_logits = views[3] if self.ids is not None else None
+        self.g_u = views[4] if self.ids is not None else None
+        self.g_tok = torch.full((B,), -1, dtype=torch.int32, device=dev)
         self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
         self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
         # keep counts (row 0) and current rewards (row 1, float32 bits): one upload per boundary
@@ -327,7 +346,8 @@ class Trace:
             reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
                                   self.g_lse, self.ws_decode)
             if self.g_logits is not None:
-                reco.reco_reflect_penalty(self.g_logits, self.ids, self.g_rw, wl.tau_l, wl.tau_h, wl.beta)
+                reco.reco_penalty_sample(self.g_logits, self.ids, self.g_rw, self.g_u, self.g_tok, self.ws_sample,
+                                         wl.tau_l, wl.tau_h, wl.beta)
             if self._apool is not None:
                 self.g_slot.add_(1)
                 self.g_slot.remainder_(self.input_pool)
@@ -356,7 +376,9 @@ class Trace:
                 self.g_vn.copy_(vn)
                 if self.g_logits is not None:
                     self.g_logits.copy_(self.active_logits(t))
+                    self.g_u.copy_(self.active_draws(t))
             self.graph.replay()
+            self.tokens = self.g_tok
             return self.g_out, self.g_lse, self.g_logits
         q, kn, vn = self.active_inputs(t)
         out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
@@ -366,7 +388,9 @@ class Trace:
         if self.ids is not None:
             logits = self.active_logits(t)
             rw = self.staging.put([self.current_reward(s) for s in self.active], torch.float32)
-            reco.reco_reflect_penalty(logits, self.ids, rw, wl.tau_l, wl.tau_h, wl.beta)
+            self.tokens = torch.empty(len(self.active), dtype=torch.int32, device=self.device)
+            reco.reco_penalty_sample(logits, self.ids, rw, self.active_draws(t), self.tokens, self.ws_sample,
+                                     wl.tau_l, wl.tau_h, wl.beta)
         return out, lse, logits
 
     def run(self, max_tokens=None, on_token=None, on_boundary=None) -> TraceEvents:

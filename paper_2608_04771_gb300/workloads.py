@@ -191,6 +191,12 @@ def make_vocab_logits(wl: Workload, device="cpu", stream: int = 5) -> torch.Tens
     return randn((wl.batch, wl.vocab), wl, stream, device, torch.float32) * 2.0
 
 
+def make_draws(wl: Workload, n: int, stream: int = 13) -> np.ndarray:
+    """[n] float32 uniform draws on the 2^-24 grid of [0, 1) (exact in float32)."""
+    rng = _np_rng(wl, stream)
+    return (rng.integers(0, 1 << 24, n) / float(1 << 24)).astype(np.float32)
+
+
 def make_reflection_ids(wl: Workload) -> np.ndarray:
     rng = _np_rng(wl, 6)
     return rng.choice(wl.vocab, wl.n_ids, replace=False).astype(np.int32)

@@ -95,3 +95,24 @@ def assert_kept_match(gpu_idx: np.ndarray, ora_idx: np.ndarray, ora_scores: np.n
         assert j < L - w and abs(cand[j] - sk) <= TIE_RTOL * abs(sk), \
             f"{what}: index {j} differs with score {cand[j]!r} vs boundary {sk!r}"
     return len(diff)
+
+
+SAMPLE_EPS = 1e-5  # draws this close to a CDF boundary may take the neighbouring token
+
+
+def assert_tokens_valid(got, zp, u, ref, max_inexact):
+    """Sampled tokens vs the oracle's draw: equal, or (a draw within SAMPLE_EPS of a boundary of
+    the cumulative distribution) between the oracle's tokens at u -/+ SAMPLE_EPS and with mass.
+    zp: the penalised logits [B, V]; at most max_inexact rows may differ."""
+    got = np.asarray(got)
+    B = got.shape[0]
+    none = np.zeros(0, np.int32)
+    zero = np.zeros(B, np.float32)
+    _, t_lo, _, _, _ = oracle.penalty_sample(zp, none, zero, (np.asarray(u) - SAMPLE_EPS).astype(np.float32))
+    _, t_hi, _, _, _ = oracle.penalty_sample(zp, none, zero, (np.asarray(u) + SAMPLE_EPS).astype(np.float32))
+    exact = got == ref
+    has_mass = np.array([g >= 0 and zp[b, g] != -np.inf for b, g in enumerate(got)])
+    near = (got >= t_lo) & (got <= t_hi) & has_mass
+    bad = np.nonzero(~(exact | near))[0]
+    assert bad.size == 0, [(b, got[b], ref[b], t_lo[b], t_hi[b]) for b in bad[:5]]
+    assert (~exact).sum() <= max_inexact, int((~exact).sum())

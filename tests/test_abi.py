@@ -91,6 +91,11 @@ def test_workspace_sizes(L):
     assert reco.reco_workspace_bytes(reco.RECO_OP_SELECT, kv) >= units * 100 * 4
     assert reco.reco_workspace_bytes(reco.RECO_OP_DECODE, kv) > 0
     assert reco.reco_workspace_bytes(reco.RECO_OP_PPL, None, 64) == 256
+    # sampling: (max, sum) float pairs per 4096-logit segment of one row
+    assert reco.reco_workspace_bytes(reco.RECO_OP_SAMPLE, None, 152064) == 38 * 8
+    assert reco.reco_workspace_bytes(reco.RECO_OP_SAMPLE, None, 1) == 8
+    with pytest.raises(reco.RecoError):
+        reco.reco_workspace_bytes(reco.RECO_OP_SAMPLE, None, 0)
     with pytest.raises(reco.RecoError):
         reco.reco_workspace_bytes(reco.RECO_OP_SCORE, _kv(d=96), 16)
     with pytest.raises(reco.RecoError):
@@ -122,3 +127,22 @@ def test_device_calls_validate_before_launch(L):
     assert st == reco.RECO_EINVAL
     st = L.reco_answer_ppl(vp(16), vp(16), None, 2, 4, 10, 1.1, vp(16), vp(16), None, 0, None)
     assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+
+
+def test_penalty_sample_validates_before_launch(L):
+    vp = ctypes.c_void_p
+    ws = vp(256 * 1000)
+    args = dict(logits=vp(256), B=4, V=1000, ids=vp(512), n_ids=2, rewards=vp(768), tau_l=0.4, tau_h=0.8, beta=4.0,
+                uniforms=vp(1024), tokens=vp(1280), beta_out=None, ws=ws, ws_bytes=4 * 8, stream=None)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return L.reco_penalty_sample(a["logits"], a["B"], a["V"], a["ids"], a["n_ids"], a["rewards"], a["tau_l"],
+                                     a["tau_h"], a["beta"], a["uniforms"], a["tokens"], a["beta_out"], a["ws"],
+                                     a["ws_bytes"], a["stream"])
+    assert call(uniforms=None) == reco.RECO_EINVAL and b"NULL" in L.reco_last_error()
+    assert call(tokens=vp(1281)) == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    assert call(ws_bytes=4 * 8 - 1) == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    assert call(V=4096 * 1024 + 1) == reco.RECO_EUNSUPPORTED
+    assert call(beta=-1.0) == reco.RECO_EINVAL
+    assert call(B=0) == reco.RECO_EINVAL

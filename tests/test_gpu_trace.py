@@ -1,17 +1,18 @@
 """The step-loop trace (ragged step boundaries, compression at every boundary,
-decode between, penalty every token, answer probe on two top-band rewards, stopped
-sequences leaving the batch) replayed in lock-step by the oracle.
+decode between, penalty and a draw every token, answer probe on two top-band rewards,
+stopped sequences leaving the batch) replayed in lock-step by the oracle.
 
 The oracle keeps its own float64-computed cache state from the same seeded inputs
-(never from the GPU's results) and checks, at every token, every decode output and
-the penalised logits, and at every boundary the scores and kept sets of the
-sequences that compress, and every probe's PPL and stop decision."""
+(never from the GPU's results) and checks, at every token, every decode output, the
+penalised logits and the sampled tokens (equal up to the boundary band), at every
+boundary the scores and kept sets of the sequences that compress, and every probe's
+PPL and stop decision."""
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from helpers import DECODE_ATOL, PPL_RTOL, assert_kept_match, assert_scores_close, np32
+from helpers import DECODE_ATOL, PPL_RTOL, assert_kept_match, assert_scores_close, assert_tokens_valid, np32
 from paper_2608_04771_gb300 import reco, trace
 from paper_2608_04771_gb300 import workloads as W
 
@@ -46,6 +47,7 @@ class OracleReplay:
         self.tie_diffs = 0
         self.diverged = set()  # (seq, layer, kv head) whose kept set differed within the tie band
         self.expected_probes = set()
+        self.sampled = 0  # draws checked
 
     def on_token(self, t, tr, out, lse, logits):
         wl = self.wl
@@ -75,6 +77,10 @@ class OracleReplay:
                 rw = np.array([self.hist[s][-1] if self.hist[s] else 0.0 for s in act], np.float32)
                 ref, _, _ = oracle.reflect_penalty(z, self.ids, rw, wl.tau_l, wl.tau_h, wl.beta)
                 np.testing.assert_array_equal(logits[pos].cpu().numpy().view(np.uint32), ref.view(np.uint32))
+                u = tr.token_draws(t).cpu().numpy()[act]
+                _, tref, _, _, _ = oracle.penalty_sample(z, self.ids, rw, u, wl.tau_l, wl.tau_h, wl.beta)
+                assert_tokens_valid(tr.tokens[pos].cpu().numpy(), ref, u, tref, max_inexact=1)
+                self.sampled += len(act)
             self.checked_tokens += 1
 
     def on_boundary(self, t, tr, done, keep, q_win):
