@@ -157,7 +157,9 @@ reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t 
  *   k_new, v_new : [n_layers][B][H_kv][d], cache dtype (device) or both NULL
  *   out          : [n_layers][B][H_q][d] of out_dtype (RECO_F32 or RECO_BF16)
  *   lse          : [n_layers][B][H_q] float32 or NULL
- *   ws           : workspace of reco_workspace_bytes(RECO_OP_DECODE, kv, 0) bytes
+ *   ws           : workspace of reco_workspace_bytes(RECO_OP_DECODE, kv, 0) bytes,
+ *                  zero-filled before its first use (e.g. cudaMemset); every call
+ *                  leaves its counters zero again, so it can be reused as it is
  * A unit with a length outside [0, L_cap] (or no room to append) writes zeros
  * and lse = -inf, and sets the device error word.                              */
 reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,

@@ -13,7 +13,8 @@
 // and K sides (and on the V and output sides) so that each thread's fragments are
 // whole 16-byte chunks, and the swizzle makes every fragment read conflict-free.  A unit split over several items writes partial
 // (max, sum, output) triples; the last item to finish (atomic ticket, no waiting)
-// merges them.  The appended token (k_new, v_new) is read from the inputs and written
+// merges them.  The counters live in the caller's workspace, zero-filled before its
+// first use; each launch clears what it counted, so no reset runs between launches.  The appended token (k_new, v_new) is read from the inputs and written
 // into the cache by the warp that covers its index; the last warp of the grid to
 // finish advances lens.
 //
@@ -664,6 +665,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             old = __shfl_sync(0xffffffffu, old, 0);
             __syncwarp();
             if (old == nsplit - 1) {  // last item of this unit: merge the partials
+                if (lane == 0) a.counters[2 + u] = 0;  // every piece has counted: clear for the next launch
                 // pass 1: per-query-head maxima, lanes over splits (independent loads)
                 float Mq[8];
 #pragma unroll
@@ -736,29 +738,44 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             pblk = 0;
         }
     }
-    if (aborted) return;
-    // the last warp of the grid advances the lengths (every plan has been read by then)
+    // Every warp, stopped early or not, counts itself done (a stopped one marks that
+    // first).  The last one has every other warp behind it: it advances the lengths
+    // (every plan has been read by then) and clears the counters, so a launch leaves the
+    // workspace's counters zero as it found them, also after a stop.
     int done = 0;
     __syncwarp();
-    if (lane == 0) done = atom_add_acq_rel(&a.counters[1], 1);
+    if (lane == 0) {
+        if (aborted) atomicOr(&a.counters[0], 1);
+        done = atom_add_acq_rel(&a.counters[1], 1);
+    }
     done = __shfl_sync(0xffffffffu, done, 0);
     __syncwarp();
-    if (done == total_warps - 1 && a.append) {
-        // 16 independent loads per lane in flight before any store: a few L2 round trips
-        // for the whole grid instead of one per 32 units
-        constexpr int BATCH = 16;
-        for (int u0 = 0; u0 < units; u0 += 32 * BATCH) {
-            int L[BATCH];
+    if (done == total_warps - 1) {
+        const bool any_stop = __ldcg(&a.counters[0]) != 0;
+        if (any_stop) {  // tickets of units whose pieces stopped early may still count
+            for (int u = lane; u < units; u += 32) a.counters[2 + u] = 0;
+        } else if (a.append) {
+            // 16 independent loads per lane in flight before any store: a few L2 round
+            // trips for the whole grid instead of one per 32 units
+            constexpr int BATCH = 16;
+            for (int u0 = 0; u0 < units; u0 += 32 * BATCH) {
+                int L[BATCH];
 #pragma unroll
-            for (int k = 0; k < BATCH; ++k) {
-                const int u = u0 + 32 * k + lane;
-                L[k] = u < units ? __ldcg(a.lens + u) : -1;
-            }
+                for (int k = 0; k < BATCH; ++k) {
+                    const int u = u0 + 32 * k + lane;
+                    L[k] = u < units ? __ldcg(a.lens + u) : -1;
+                }
 #pragma unroll
-            for (int k = 0; k < BATCH; ++k) {
-                const int u = u0 + 32 * k + lane;
-                if (u < units && unit_ok(L[k], a.L_cap, a.append)) a.lens[u] = L[k] + 1;
+                for (int k = 0; k < BATCH; ++k) {
+                    const int u = u0 + 32 * k + lane;
+                    if (u < units && unit_ok(L[k], a.L_cap, a.append)) a.lens[u] = L[k] + 1;
+                }
             }
+        }
+        __syncwarp();
+        if (lane == 0) {
+            a.counters[0] = 0;
+            a.counters[1] = 0;
         }
     }
 }
@@ -802,8 +819,8 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31) && slots_fit) {
         CUtensorMap mk, mv;
         if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {
-            cudaError_t e = cudaMemsetAsync(ws.counters, 0, (size_t)(2 + a.units) * 4, s);
-            if (e != cudaSuccess) return e;
+            // the counters are zero on entry (zero-filled workspace) and every launch leaves them so
+            cudaError_t e;
             const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(a.units) : tma_smem_bytes<128>(a.units);
             const void *fn = kv.d == 64 ? (const void *)decode_tma<64> : (const void *)decode_tma<128>;
             e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

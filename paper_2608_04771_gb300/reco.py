@@ -146,8 +146,9 @@ def reco_workspace_bytes(op: int, kv: reco_kv | None, w: int = 0) -> int:
 
 
 def workspace(op: int, kv: reco_kv | None, w: int = 0, device="cuda") -> torch.Tensor:
+    """A zero-filled workspace (the decode call needs its counters zero before first use)."""
     n = reco_workspace_bytes(op, kv, w)
-    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+    return torch.zeros(max(n, 256), dtype=torch.uint8, device=device)
 
 
 def reco_check(stream=None):

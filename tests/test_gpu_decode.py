@@ -114,3 +114,29 @@ def test_empty_unit_and_no_room():
     assert e.value.status == reco.RECO_EDEVICE
     assert torch.all(out[0, 0] == 0) and int(lens[0, 0, 0]) == 64 and int(lens[0, 1, 0]) == 11
     reco.reco_check()
+
+
+def test_workspace_counters_left_zero_and_reused():
+    """Units long enough to be cut between warps (their pieces merge through per-unit
+    tickets): two appends in a row on one zero-filled workspace, each checked against the
+    oracle, and the counter region is zero again after each call."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=2, L=6000, decode_steps=4)
+    K, V = W.make_cache(wl, DEV, canary=False)
+    lens_np = np.array([[[6000, 5000, 4100, 3000], [2500, 6000, 5900, 17]]] * 2, np.int32)
+    lens = torch.from_numpy(lens_np).to(DEV)
+    kv = reco.make_kv(K, V, wl.h_q)
+    ws = reco.workspace(reco.RECO_OP_DECODE, kv, 0, DEV)
+    units = wl.layers * wl.batch * wl.h_kv
+    K_np, V_np = np32(K), np32(V)
+    for step in range(2):
+        q, kn, vn = W.make_decode_step(wl, 10 + step, DEV)
+        out = torch.empty(q.shape, dtype=torch.float32, device=DEV)
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+        reco.reco_decode_attn(kv, q, kn, vn, lens, wl.scale(), out, lse, ws)
+        reco.reco_check()
+        ref, lse_ref, K_np, V_np, lens_np = _oracle_decode(wl, K_np, V_np, lens_np, np32(q), np32(kn), np32(vn))
+        assert (np.abs(out.cpu().numpy() - ref) <= DECODE_ATOL["bf16"]).all(), step
+        assert np.abs(lse.cpu().numpy() - lse_ref).max() < 1e-3
+        np.testing.assert_array_equal(lens.cpu().numpy(), lens_np)
+        counters = ws[: (2 + units) * 4].view(torch.int32).cpu().numpy()
+        assert (counters == 0).all(), counters
