@@ -2,7 +2,7 @@
 // attention whose cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2).
 //
 // bf16 path (decode_tma): a persistent split-K flash-decode, one CTA of 8 warps per
-// SM.  Every CTA first builds the same work plan from lens: the prefix sum of 16-key
+// SM (for long work 4 of them, each with a ring twice as deep).  Every CTA first builds the same work plan from lens: the prefix sum of 16-key
 // blocks per unit, with the blocks of all units laid end to end and cut into one equal
 // contiguous range per warp (a stream-K split: balanced to one block, no work queue).
 // An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
@@ -218,6 +218,7 @@ constexpr long long kSpinLimit = 1LL << 24;  // bounded mbarrier waits (about a 
 constexpr float kLazyLog2 = 8.f;             // output rescale threshold (log2 units)
 constexpr int kMinBlocksPerWarp = 4;         // fewer working warps rather than shorter ranges
 constexpr int kMaxWholeBlocks = 16;          // units of at most this many blocks are never cut
+constexpr int kDeepBlocksPerWarp = 64;       // from this many blocks per warp, half the warps with deep rings
 
 template <int D> struct TmaLayout {
     static constexpr int HALVES = D / 64;             // 128-byte boxes per row
@@ -248,20 +249,19 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     constexpr int STAGE = LY::STAGE;
     constexpr int MT = D / 16;  // m-tiles of PV (d on M)
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    __shared__ __align__(8) uint64_t bars[NW][S];
+    __shared__ __align__(8) uint64_t bars[NW * S];  // ring stages of all warps (either partition)
     __shared__ int sm_scan[NW];
     const uint32_t raw0 = (uint32_t)__cvta_generic_to_shared(smem_raw);
     const uint32_t ring0 = (raw0 + 1023u) & ~1023u;
     int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
-    const uint32_t my_ring = ring0 + (uint32_t)wid * S * STAGE;
     if (tid == 0) {  // fetch both tensor-map descriptors while the plan is built
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
     }
     if (lane == 0) {
-        for (int s2 = 0; s2 < S; ++s2) mbar_init((uint32_t)__cvta_generic_to_shared(&bars[wid][s2]), 1);
+        for (int s2 = 0; s2 < S; ++s2) mbar_init((uint32_t)__cvta_generic_to_shared(&bars[wid * S + s2]), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         fence_async_shared();
     }
@@ -325,8 +325,17 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     __syncthreads();
     const int NB = pb[units];
     const int total_warps = gridDim.x * NW;
+    // Long work (at least kDeepBlocksPerWarp blocks per warp) runs on half the warps, each
+    // with a ring twice as deep: more bytes in flight per warp keep HBM busier once every
+    // warp has many blocks; short work keeps all warps for latency.  The CTA's ring is the
+    // same either way (NW * S stages).
+    const bool deep = NB >= kDeepBlocksPerWarp * total_warps;
+    bool aborted = false;
+    {
+    const int NWm = deep ? NW / 2 : NW, Sm = deep ? 2 * S : S;  // NWm * Sm == NW * S either way
+    const uint32_t my_ring = ring0 + (uint32_t)wid * Sm * STAGE;
     // working warps: every one gets at least kMinBlocksPerWarp blocks (or all warps work)
-    const int W = max(1, min(total_warps, NB / kMinBlocksPerWarp));
+    const int W = max(1, min(NWm * (int)gridDim.x, NB / kMinBlocksPerWarp));
     const int g = lane >> 2, c = lane & 3;
     const bool out_bf16 = a.out_bf16 != 0;
     auto wstart = [&](int w) { return (int)((long long)w * NB / W); };  // ideal first block of warp w
@@ -432,6 +441,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // item into the next one (grabbed one item ahead) so no refill bubble opens between
     // items; the warp consumes blocks in issue order.
     uint32_t issued = 0, consumed = 0;
+    uint32_t p_slot = 0, c_slot = 0, c_par = 0;  // ring slot of the next issue / next wait, wait phase
     Item cur = next_item();
     uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
     if (cur.nblk >= 0) load_q(cur, qa_n);
@@ -439,7 +449,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     Item pit = cur;  // item the producer is issuing from
     int pblk = 0;
     bool p_on_next = false;
-    bool aborted = false;
     auto can_issue = [&]() {
         if (pblk < pit.nblk) return true;
         if (!p_on_next && nxt.nblk > 0) {
@@ -451,9 +460,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         return false;
     };
     auto issue = [&]() {
-        const uint32_t slot = issued % S;
+        const uint32_t slot = p_slot;
         if (lane == 0) {
-            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
+            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid * Sm + slot]);
             const uint32_t dst = my_ring + slot * STAGE;
             const int y = pit.u * a.L_cap + pit.k0 + 16 * pblk;
             fence_async_shared();
@@ -466,6 +475,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         ++pblk;
         ++issued;
+        if (++p_slot == (uint32_t)Sm) p_slot = 0;
     };
 
     while (cur.nblk >= 0) {
@@ -481,7 +491,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 
         // start this item's copies before the wait on its query registers below
         __syncwarp();
-        while (issued - consumed < (uint32_t)S && can_issue()) issue();
+        while (issued - consumed < (uint32_t)Sm && can_issue()) issue();
         uint32_t qa[D / 16][2];
 #pragma unroll
         for (int j = 0; j < D / 16; ++j) {
@@ -496,14 +506,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 
         for (int bi = 0; bi < cur.nblk; ++bi) {
             __syncwarp();
-            while (issued - consumed < (uint32_t)S && can_issue()) issue();
-            const uint32_t slot = consumed % S;
-            const uint32_t parity = (consumed / S) & 1u;
-            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid][slot]);
+            while (issued - consumed < (uint32_t)Sm && can_issue()) issue();
+            const uint32_t slot = c_slot, parity = c_par;
+            const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid * Sm + slot]);
             if (!mbar_wait_bounded(bar, parity, kSpinLimit)) {  // a copy never landed: report, drain, stop
                 if (lane == 0) raise_error(a.err, ERR_INTERNAL);
                 for (uint32_t q2 = consumed + 1; q2 < issued; ++q2)
-                    mbar_wait_bounded((uint32_t)__cvta_generic_to_shared(&bars[wid][q2 % S]), (q2 / S) & 1u,
+                    mbar_wait_bounded((uint32_t)__cvta_generic_to_shared(&bars[wid * Sm + q2 % Sm]), (q2 / Sm) & 1u,
                                       kSpinLimit);
                 aborted = true;
                 break;
@@ -603,6 +612,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 }
             }
             ++consumed;
+            if (++c_slot == (uint32_t)Sm) {
+                c_slot = 0;
+                c_par ^= 1u;
+            }
         }
         if (aborted) break;
 
@@ -738,6 +751,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             pblk = 0;
         }
     }
+    }
+
     // Every warp, stopped early or not, counts itself done (a stopped one marks that
     // first).  The last one has every other warp behind it: it advances the lengths
     // (every plan has been read by then) and clears the counters, so a launch leaves the
