@@ -15,23 +15,50 @@
 
 namespace reco {
 
+// The ids of R in shared memory (one coalesced read per CTA), so the duplicate check of
+// each id against the ones before it runs on shared memory; longer lists are read
+// from global memory.
+constexpr int kIdsShared = 1024;
+
+__device__ __forceinline__ bool stage_ids(const int32_t *__restrict__ ids, int n_ids, int *sm_ids)
+{
+    const bool staged = n_ids <= kIdsShared;  // uniform across the CTA
+    if (staged) {
+        for (int i = threadIdx.x; i < n_ids; i += blockDim.x) sm_ids[i] = ids[i];
+        __syncthreads();
+    }
+    return staged;
+}
+
+__device__ __forceinline__ bool seen_before(const int32_t *__restrict__ ids, const int *sm_ids, bool staged, int i,
+                                            int id)
+{
+    bool dup = false;
+    if (staged) {
+        for (int k = 0; k < i; ++k) dup |= sm_ids[k] == id;
+    } else {
+        for (int k = 0; k < i && !dup; ++k) dup = ids[k] == id;
+    }
+    return dup;
+}
+
 __global__ void reflect_penalty_kernel(float *logits, int V, const int32_t *__restrict__ ids, int n_ids,
                                        const float *__restrict__ rewards, float tau_l, float tau_h,
                                        float beta, float *beta_out, unsigned *err)
 {
+    __shared__ int sm_ids[kIdsShared];
     const int b = blockIdx.x;
     const float v = rewards[b];
     const float bi = (v <= tau_l) ? 0.f : ((v >= tau_h) ? beta : beta * 0.5f);
     if (threadIdx.x == 0 && beta_out) beta_out[b] = bi;
+    const bool staged = stage_ids(ids, n_ids, sm_ids);
     for (int i = threadIdx.x; i < n_ids; i += blockDim.x) {
-        const int id = ids[i];
+        const int id = staged ? sm_ids[i] : ids[i];
         if (id < 0 || id >= V) {
             if (b == 0) raise_error(err, ERR_ID);
             continue;
         }
-        bool dup = false;
-        for (int k = 0; k < i && !dup; ++k) dup = ids[k] == id;
-        if (dup || bi == 0.f) continue;
+        if (bi == 0.f || seen_before(ids, sm_ids, staged, i, id)) continue;
         float *p = logits + (size_t)b * V + id;
         *p = __fsub_rn(*p, bi);
     }
@@ -61,22 +88,22 @@ __global__ void __launch_bounds__(NT) sample_segments(float *__restrict__ logits
 {
     constexpr int PER = kSampleSeg / NT;
     __shared__ float sm_m[NT / 32], sm_s[NT / 32];
+    __shared__ int sm_ids[kIdsShared];
     const int sg = blockIdx.x, b = blockIdx.y;
     const int lo = sg * kSampleSeg, hi = min(V, lo + kSampleSeg);
     float *z = logits + (size_t)b * V;
     const float v = rewards[b];
     const float bi = (v <= tau_l) ? 0.f : ((v >= tau_h) ? beta : beta * 0.5f);
     if (sg == 0 && threadIdx.x == 0 && beta_out) beta_out[b] = bi;
+    const bool staged = stage_ids(ids, n_ids, sm_ids);
     for (int i = threadIdx.x; i < n_ids; i += NT) {
-        const int id = ids[i];
+        const int id = staged ? sm_ids[i] : ids[i];
         if (id < 0 || id >= V) {
             if (b == 0 && sg == 0) raise_error(err, ERR_ID);
             continue;
         }
         if (id < lo || id >= hi || bi == 0.f) continue;
-        bool dup = false;
-        for (int k = 0; k < i && !dup; ++k) dup = ids[k] == id;
-        if (!dup) z[id] = __fsub_rn(z[id], bi);
+        if (!seen_before(ids, sm_ids, staged, i, id)) z[id] = __fsub_rn(z[id], bi);
     }
     __syncthreads();  // the segment's penalised logits are visible to the whole CTA
     float y[PER];
