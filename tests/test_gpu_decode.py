@@ -140,3 +140,25 @@ def test_workspace_counters_left_zero_and_reused():
         np.testing.assert_array_equal(lens.cpu().numpy(), lens_np)
         counters = ws[: (2 + units) * 4].view(torch.int32).cpu().numpy()
         assert (counters == 0).all(), counters
+
+
+def test_deep_ring_partition_ragged():
+    """About 96 K blocks of 16 keys: the launch runs 4 warps per CTA with rings twice as deep.
+    Ragged lengths (long units cut between warps, short ones whole), two appends in a row."""
+    wl = W.WORKLOADS["7b"].reduced(layers=4, batch=8, L=12000, decode_steps=4)
+    rng = np.random.default_rng(41)
+    lens = rng.integers(9000, 12001, (4, 8, wl.h_kv)).astype(np.int32)
+    lens[0, 0, :] = [1, 17, 255, 256]  # short units among the long ones
+    assert (lens.astype(np.int64) + 15).__floordiv__(16).sum() >= 64 * 152 * 8
+    _check(wl, lens, True, steps=2)
+
+
+@pytest.mark.parametrize("shape", [(64, 16, 56, 8), (1, 8193, 7, 1)])
+def test_tma_path_unit_limit(shape):
+    """8192 units (the most the TMA path plans in shared memory) and 8193 (the SIMT path)."""
+    layers, batch, h_q, h_kv = shape
+    wl = W.WORKLOADS["7b"].reduced(layers=layers, batch=batch, h_q=h_q, h_kv=h_kv, L=40, decode_steps=4)
+    rng = np.random.default_rng(42 + layers)
+    lens = rng.integers(1, 41, (layers, batch, h_kv)).astype(np.int32)
+    assert lens.size in (8192, 8193)
+    _check(wl, lens, True)

@@ -201,3 +201,12 @@ def test_penalty_sample_bad_id_sets_device_error():
     ref, _, _ = oracle.reflect_penalty(np.zeros((2, 10), np.float32), [3, 10, -1], [1.0, 0.5])
     np.testing.assert_array_equal(z.cpu().numpy(), ref)
     reco.reco_check()
+
+
+def test_penalty_sample_largest_vocab():
+    """V = 4 * 1024 * 1024 logits per row (1024 segments, the most a row may have)."""
+    V, B = 4 * 1024 * 1024, 2
+    rng = np.random.default_rng(35)
+    z = torch.from_numpy((rng.standard_normal((B, V)) * 2).astype(np.float32)).to(DEV)
+    ids_np = rng.choice(V, 16, replace=False).astype(np.int32)
+    _sample_case(z, ids_np, np.array([1.0, 0.6], np.float32), np.array([0.37, 0.999], np.float32), max_inexact=1)
