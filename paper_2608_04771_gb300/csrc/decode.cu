@@ -443,9 +443,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     uint32_t issued = 0, consumed = 0;
     uint32_t p_slot = 0, c_slot = 0, c_par = 0;  // ring slot of the next issue / next wait, wait phase
     Item cur = next_item();
-    uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
-    if (cur.nblk >= 0) load_q(cur, qa_n);
-    Item nxt = cur.nblk >= 0 ? next_item() : cur;
+    Item nxt;
+    nxt.nblk = -1;  // looked up below, after the first copies are out
     Item pit = cur;  // item the producer is issuing from
     int pblk = 0;
     bool p_on_next = false;
@@ -477,6 +476,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         ++issued;
         if (++p_slot == (uint32_t)Sm) p_slot = 0;
     };
+    // the first piece's copies go out before the next piece is looked up (that lookup
+    // reads a length from global memory)
+    __syncwarp();
+    while (issued < (uint32_t)Sm && pblk < pit.nblk) issue();
+    uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
+    if (cur.nblk >= 0) load_q(cur, qa_n);
+    nxt = cur.nblk >= 0 ? next_item() : cur;
 
     while (cur.nblk >= 0) {
         const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
