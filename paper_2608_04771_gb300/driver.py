@@ -74,7 +74,7 @@ class HotPath:
     def compress(self, stream=None):
         wl = self.wl
         reco.reco_score_cache(self.kv, self.q_win, self.lens, wl.w, wl.pool, wl.scale(), self.scores,
-                              self.ws_score, stream)
+                              self.ws_score, stream=stream)
         reco.reco_select_compact(self.kv, self.scores, self.lens, self.keep, wl.w, self.kept,
                                  self.ws_select, stream)
 
