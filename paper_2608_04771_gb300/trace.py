@@ -340,9 +340,10 @@ class Trace:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="relaxed"):
             if self._apool is not None:
-                # 8-byte elements: every part is a multiple of 256 bytes
-                torch.index_select(self._apool.view(torch.int64), 0, self.g_slot,
-                                   out=self.g_in.view(torch.int64).view(1, -1))
+                # 16-byte elements (every part is a multiple of 256 bytes): a quarter
+                # fewer nanoseconds than 8-byte ones for the same bytes
+                torch.index_select(self._apool.view(torch.complex128), 0, self.g_slot,
+                                   out=self.g_in.view(torch.complex128).view(1, -1))
             reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
                                   self.g_lse, self.ws_decode)
             if self.g_logits is not None:
