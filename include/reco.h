@@ -4,13 +4,16 @@
  * Reasoning": reward-set retention (Eq. 1), attention-guided cache scoring
  * (Eq. 2), per-head top-m selection with in-place compaction (Sec. 3.2), decode
  * attention over the ragged compacted cache, the reward-banded reflection
- * penalty (Eq. 3-4) and the answer-perplexity stop test (Eq. 5-6).
+ * penalty (Eq. 3-4) with the draw of the next token from the penalised logits
+ * (Sec. 3.3), and the answer-perplexity stop test (Eq. 5-6).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
  *  - Pointers are DEVICE pointers owned by the caller unless marked "host".
  *    The library never allocates device memory: calls that need scratch take a
- *    caller-owned workspace sized by reco_workspace_bytes().
+ *    caller-owned workspace sized by reco_workspace_bytes() (the decode's must
+ *    be zero-filled before its first use; each call leaves it reusable), except
+ *    reco_answer_ppl_static, which uses a fixed array inside the library.
  *  - Device calls are asynchronous on the given stream and return after the
  *    launches are queued.  They return RECO_OK, or an error status before
  *    launching anything when a host-side check fails (nothing is modified then).
@@ -159,7 +162,8 @@ reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t 
  *   lse          : [n_layers][B][H_q] float32 or NULL
  *   ws           : workspace of reco_workspace_bytes(RECO_OP_DECODE, kv, 0) bytes,
  *                  zero-filled before its first use (e.g. cudaMemset); every call
- *                  leaves its counters zero again, so it can be reused as it is
+ *                  leaves its counters zero again, so it can be reused as it is;
+ *                  calls sharing one workspace must not overlap on the GPU
  * A unit with a length outside [0, L_cap] (or no room to append) writes zeros
  * and lse = -inf, and sets the device error word.                              */
 reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,
