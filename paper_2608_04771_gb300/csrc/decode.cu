@@ -39,10 +39,10 @@ DecodeWs decode_ws_layout(const reco_kv &kv, void *base)
         return r;
     };
     DecodeWs ws;
-    ws.max_items = kDecodeMaxTarget + (int)units;
+    ws.part_slots = kDecodePartSlots;
     ws.counters = (int32_t *)take((2 + units) * 4);
-    ws.part_ml = (float *)take((size_t)ws.max_items * G * 2 * 4);
-    ws.part_o = (float *)take((size_t)ws.max_items * G * kv.d * 4);
+    ws.part_ml = (float *)take((size_t)ws.part_slots * G * 2 * 4);
+    ws.part_o = (float *)take((size_t)ws.part_slots * G * kv.d * 4);
     ws.bytes = off;
     return ws;
 }
@@ -59,7 +59,7 @@ struct DecodeArgs {
     int32_t *counters;
     float *part_ml;
     float *part_o;
-    int units, Hq, Hkv, G, L_cap, max_items, append, out_bf16;
+    int units, Hq, Hkv, G, L_cap, append, out_bf16;
     float c2;  // scale * log2(e)
     unsigned *err;
 };
@@ -829,14 +829,13 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.Hkv = kv.H_kv;
     a.G = kv.H_q / kv.H_kv;
     a.L_cap = kv.L_cap;
-    a.max_items = ws.max_items;
     a.append = (k_new && v_new) ? 1 : 0;
     a.out_bf16 = out_dtype == RECO_BF16 ? 1 : 0;
     a.c2 = scale * kLog2e;
     a.err = err;
     const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
     // partial slots: two per warp of the grid
-    const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.max_items;
+    const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.part_slots;
     if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31) && slots_fit) {
         CUtensorMap mk, mv;
         if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {

@@ -10,8 +10,10 @@ namespace reco {
 
 // Keys per scoring work item (one CTA per (unit, chunk) in both scoring passes).
 constexpr int kScoreChunk = 2048;
-// Upper bound on decode split-K work items beyond one per unit.
-constexpr int kDecodeMaxTarget = 16384;
+// Decode (m, l, O) partial slots in the workspace: two per warp of a grid of up to
+// 256 SMs x 8 warps (the workspace size may not depend on the device; a larger grid
+// takes the SIMT path).
+constexpr int kDecodePartSlots = 4096;
 // Sampling: logits per pass-1 segment, and the most segments a row may have.
 constexpr int kSampleSeg = 4096;
 constexpr int kSampleMaxSeg = 1024;
@@ -50,10 +52,10 @@ struct SelectWs {
 };
 
 struct DecodeWs {
-    int32_t *counters;  // [2 + units]: work counter, finished warps, per-unit tickets
-    float *part_ml;     // [max_items][G][2]  (m log2, l)
-    float *part_o;      // [max_items][G][d]  unnormalised output
-    int max_items;
+    int32_t *counters;  // [2 + units]: [0] a warp stopped early, [1] finished warps, [2 + u] merge tickets
+    float *part_ml;     // [part_slots][G][2]  (m log2, l)
+    float *part_o;      // [part_slots][G][d]  unnormalised output
+    int part_slots;
     size_t bytes;
 };
 
