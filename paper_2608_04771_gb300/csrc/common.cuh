@@ -31,6 +31,31 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(f
     return __float2bfloat16_rn(x);
 }
 
+// Programmatic dependent launch.  Kernels launched with launch_pdl() may be scheduled
+// while the previous kernel in the stream drains; each one calls wait_prior_grid()
+// before it reads anything a previous kernel wrote (it returns at once when the launch
+// was an ordinary one).  No kernel signals its dependents early, so a dependent grid
+// starts only as the previous one's blocks exit: what overlaps is launch processing and
+// the part of a kernel before its wait.
+__device__ __forceinline__ void wait_prior_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // 2^x on the MUFU pipe (ex2.approx.ftz.f32).
 __device__ __forceinline__ float fast_exp2(float x)
 {

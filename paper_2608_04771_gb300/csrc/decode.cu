@@ -256,7 +256,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int units = a.units;
-    if (tid == 0) {  // fetch both tensor-map descriptors while the plan is built
+    if (tid == 0) {  // fetch both tensor-map descriptors (kernel parameters) while the previous kernel drains
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
     }
@@ -266,6 +266,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         fence_async_shared();
     }
     __syncwarp();
+    wait_prior_grid();  // lens, q and the new rows may come from the previous kernels
 
     // ---- plan: identical in every CTA (lens are not modified until every warp is done).
     // Each unit's keys form nb_u = ceil(le_u / 16) blocks; the blocks of all units are laid
@@ -847,10 +848,10 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
             if (e != cudaSuccess) return e;
             const int grid = device_sm_count();
             if (kv.d == 64)
-                decode_tma<64><<<grid, kDecodeWarps * 32, smem, s>>>(mk, mv, a);
+                e = launch_pdl(decode_tma<64>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, a);
             else
-                decode_tma<128><<<grid, kDecodeWarps * 32, smem, s>>>(mk, mv, a);
-            return cudaGetLastError();
+                e = launch_pdl(decode_tma<128>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, a);
+            return e != cudaSuccess ? e : cudaGetLastError();
         }
     }
     const unsigned grid = (unsigned)a.units;

@@ -47,6 +47,7 @@ __global__ void reflect_penalty_kernel(float *logits, int V, const int32_t *__re
                                        float beta, float *beta_out, unsigned *err)
 {
     __shared__ int sm_ids[kIdsShared];
+    wait_prior_grid();
     const int b = blockIdx.x;
     const float v = rewards[b];
     const float bi = (v <= tau_l) ? 0.f : ((v >= tau_h) ? beta : beta * 0.5f);
@@ -69,9 +70,8 @@ cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int 
                            unsigned *err, cudaStream_t s)
 {
     int nt = n_ids < 32 ? 32 : (n_ids > 256 ? 256 : ((n_ids + 31) / 32) * 32);
-    reflect_penalty_kernel<<<B, nt, 0, s>>>(logits, V, ids, n_ids, rewards, tau_l, tau_h, beta, beta_out,
-                                            err);
-    return cudaGetLastError();
+    return launch_pdl(reflect_penalty_kernel, dim3(B), dim3(nt), 0, s, logits, V, ids, n_ids, rewards, tau_l, tau_h,
+                      beta, beta_out, err);
 }
 
 // ---------------------------------------------------------------- penalty + sampling
@@ -89,6 +89,7 @@ __global__ void __launch_bounds__(NT) sample_segments(float *__restrict__ logits
     constexpr int PER = kSampleSeg / NT;
     __shared__ float sm_m[NT / 32], sm_s[NT / 32];
     __shared__ int sm_ids[kIdsShared];
+    wait_prior_grid();
     const int sg = blockIdx.x, b = blockIdx.y;
     const int lo = sg * kSampleSeg, hi = min(V, lo + kSampleSeg);
     float *z = logits + (size_t)b * V;
@@ -224,6 +225,7 @@ __global__ void __launch_bounds__(NT) sample_pick(const float *__restrict__ logi
     __shared__ float sm_w[NT / 32];
     __shared__ float sm_f[1];
     __shared__ int sm_i[2];
+    wait_prior_grid();
     const int b = blockIdx.x, tid = threadIdx.x;
     const float2 *pp = part + (size_t)b * nseg;
     float2 q[SR];
@@ -285,12 +287,11 @@ cudaError_t launch_penalty_sample(float *logits, int B, int V, const int32_t *id
                                   float *beta_out, float2 *part, unsigned *err, cudaStream_t s)
 {
     const int nseg = (V + kSampleSeg - 1) / kSampleSeg;
-    sample_segments<256><<<dim3(nseg, B), 256, 0, s>>>(logits, V, nseg, ids, n_ids, rewards, tau_l, tau_h, beta,
-                                                      beta_out, part, err);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(sample_segments<256>, dim3(nseg, B), dim3(256), 0, s, logits, V, nseg, ids, n_ids,
+                               rewards, tau_l, tau_h, beta, beta_out, part, err);
     if (e != cudaSuccess) return e;
-    sample_pick<256><<<B, 256, 0, s>>>(logits, V, nseg, uniforms, part, tokens);
-    return cudaGetLastError();
+    return launch_pdl(sample_pick<256>, dim3(B), dim3(256), 0, s, (const float *)logits, V, nseg, uniforms,
+                      (const float2 *)part, tokens);
 }
 
 // Online (max, sum) in the log2 domain over four values.
