@@ -268,6 +268,74 @@ def workload_name(wl):
 
 
 # ------------------------------------------------------------------ GPU arm
+def time_penalty(hp, n=128, reps=4):
+    """reco_reflect_penalty on the step's logits, ids and rewards (a copy of the logits),
+    timed apart from the step so that no event pair sits between the step's launches:
+    n launches captured in one CUDA graph, the way the step issues them after each decode."""
+    from paper_2608_04771_gb300 import reco
+    wl = hp.wl
+    z = hp.logits.clone()
+    beta = torch.empty_like(hp.beta)
+    reco.reco_reflect_penalty(z, hp.ids, hp.rewards, wl.tau_l, wl.tau_h, wl.beta, beta)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="relaxed"):
+        for _ in range(n):
+            reco.reco_reflect_penalty(z, hp.ids, hp.rewards, wl.tau_l, wl.tau_h, wl.beta, beta)
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        g.replay()
+    b.record()
+    b.synchronize()
+    reco.reco_check()
+    return {"ms_per_launch": a.elapsed_time(b) / (reps * n),
+            "timing": f"{n} launches on the step's buffers captured in one CUDA graph, outside the timed step"}
+
+
+def time_score_lse(hp, alg, reps=5):
+    """Eq. 2 with the window rows' normalisers from the decode (reco_score_cache_lse) on the
+    step's pristine cache, beside the two-pass reco_score_cache, both timed apart from the
+    step.  The normalisers are the lse outputs of the library's decode of each window query
+    over the keys Eq. 2 lets it see (lens L-w+t+1, no append), as the decode of the window
+    tokens would have returned them.  Both results are compared element by element."""
+    from paper_2608_04771_gb300 import reco
+    wl, dev = hp.wl, hp.K.device
+    hp.reset()
+    ws_dec = reco.workspace(reco.RECO_OP_DECODE, hp.kv, 0, dev)
+    row_lse = torch.empty((wl.w, wl.layers, wl.batch, wl.h_q), dtype=torch.float32, device=dev)
+    out = torch.empty((wl.layers, wl.batch, wl.h_q, wl.d), dtype=torch.bfloat16, device=dev)
+    for t in range(wl.w):
+        lens_t = hp.lens0 - (wl.w - 1 - t)
+        reco.reco_decode_attn(hp.kv, hp.q_win[:, :, :, t, :].contiguous(), None, None, lens_t, wl.scale(), out,
+                              row_lse[t], ws_dec)
+    two = torch.empty_like(hp.scores)
+    one = torch.empty_like(hp.scores)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    t2, t1 = [], []
+    for _ in range(reps):
+        ev[0].record()
+        reco.reco_score_cache(hp.kv, hp.q_win, hp.lens, wl.w, wl.pool, wl.scale(), two, hp.ws_score)
+        ev[1].record()
+        reco.reco_score_cache_lse(hp.kv, hp.q_win, hp.lens, row_lse, wl.w, wl.pool, wl.scale(), one, hp.ws_score)
+        ev[2].record()
+        ev[2].synchronize()
+        t2.append(ev[0].elapsed_time(ev[1]))
+        t1.append(ev[1].elapsed_time(ev[2]))
+    reco.reco_check()
+    nc = wl.L - wl.w
+    a, b = two[..., :nc].double(), one[..., :nc].double()
+    rel = float(((a - b).abs() / a.abs().clamp_min(1e-30)).max())
+    ms1, ms2 = statistics.median(t1), statistics.median(t2)
+    k_bytes = wl.units * wl.L * wl.d * wl.elem_bytes
+    return {"ms": ms1, "two_pass_ms": ms2, "TFLOP/s": alg["score_flops"] / ms1 / 1e9,
+            "K GB/s": k_bytes / ms1 / 1e6, "max_rel_diff_vs_two_pass": rel,
+            "timing": "median of 5 calls on the pristine cache, outside the timed step; normalisers from the "
+                      "decode of each window query (no append)"}
+
+
 def time_penalty_sample(wl, dev, n_buf=32, reps=4):
     """The penalty followed by one draw per sequence (reco_penalty_sample) on the workload's
     vocabulary, timed apart from the step: n_buf logits buffers (more bytes than L2) are
@@ -322,7 +390,7 @@ def run_gpu(args, wl):
     reco.reco_check()
     torch.cuda.synchronize()
 
-    ph = {k: [] for k in ("score", "select", "decode", "penalty", "ppl", "step")}
+    ph = {k: [] for k in ("score", "select", "decode", "ppl", "step")}
     dec_ev = [(ev(), ev()) for _ in range(wl.decode_steps)]
     barrier(world)
     torch.cuda.synchronize()
@@ -335,17 +403,12 @@ def run_gpu(args, wl):
             e1.record(stream)
             reco.reco_select_compact(hp.kv, hp.scores, hp.lens, hp.keep, wl.w, hp.kept, hp.ws_select)
             e2.record(stream)
-            pen_ev = []
             for s in range(wl.decode_steps):
                 dec_ev[s][0].record(stream)
                 hp.decode(s)
                 dec_ev[s][1].record(stream)
                 if hp.has_vocab:
-                    pa, pb = ev(), ev()
-                    pa.record(stream)
                     hp.penalty()
-                    pb.record(stream)
-                    pen_ev.append((pa, pb))
             e3.record(stream)
             if hp.has_vocab:
                 hp.probe()
@@ -354,7 +417,6 @@ def run_gpu(args, wl):
             ph["score"].append(e0.elapsed_time(e1))
             ph["select"].append(e1.elapsed_time(e2))
             ph["decode"].append([a.elapsed_time(b) for a, b in dec_ev])
-            ph["penalty"].append([a.elapsed_time(b) for a, b in pen_ev])
             ph["ppl"].append(e3.elapsed_time(e4))
             ph["step"].append(e0.elapsed_time(e4))
         torch.cuda.synchronize()
@@ -380,11 +442,11 @@ def run_gpu(args, wl):
         "decode": {"ms_per_launch": dec_avg_ms, "GB/s": dec_achieved, "launches": wl.decode_steps},
     }
     if hp.has_vocab:
-        pen_ms = float(np.array(ph["penalty"]).mean())
-        kernels["penalty"] = {"ms_per_launch": pen_ms}
+        kernels["penalty"] = time_penalty(hp)
         kernels["ppl"] = {"ms": statistics.mean(ph["ppl"]),
                           "GB/s": alg["ppl_bytes"] / statistics.mean(ph["ppl"]) / 1e6}
         kernels["penalty_sample"] = time_penalty_sample(wl, dev)
+    kernels["score_lse"] = time_score_lse(hp, alg)
 
     e2e = run_e2e(hp, wl, args, world) if not args.no_e2e else None
     clocks = clk.summary()

@@ -131,6 +131,27 @@ reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t
                              int w, int pool_kernel, float scale, float *scores, void *ws, size_t ws_bytes,
                              cudaStream_t stream);
 
+/* Eq. 2 as reco_score_cache computes it, with the row normalisers of the window
+ * queries taken from the decode instead of from a first pass over the keys.  In
+ * Eq. 2 each window row is softmax_j over the keys its query may see; when the
+ * window queries are the queries of the last w decoded tokens (Sec. 3.2, the
+ * observation window), window query t of unit (layer, b, h) is the query of the
+ * token at position L-w+t, and when that token was decoded the cache held exactly
+ * its keys j <= L-w+t.  The log-sum-exp reco_decode_attn returned for that query
+ * is then the row's log normaliser, so only one pass over K remains.
+ *   row_lse: [w][n_layers][B][H_q] float32 (device): row_lse[t][layer][b][hq] =
+ *            log sum_{j <= L-w+t} exp(scale * q_win[layer,b,hq,t,:] . K[unit,j,:])
+ *            (natural log; the lse output of the reco_decode_attn call that
+ *            appended the token at position L-w+t, same scale).  The caller
+ *            vouches for that correspondence: no compression of the unit between
+ *            those decodes and this call.  A non-finite entry sets the device
+ *            error word; that row then adds nothing to the scores.
+ * Every other argument, the result and the workspace are those of
+ * reco_score_cache.                                                             */
+reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int32_t *lens, const int32_t *keep,
+                                 const float *row_lse, int w, int pool_kernel, float scale, float *scores, void *ws,
+                                 size_t ws_bytes, cudaStream_t stream);
+
 /* Top-m selection and in-place compaction (Sec. 3.2: keep the m_i best tokens,
  * the latest w always retained; compress the L cached tokens down to m_i).
  * For unit (layer, b, h) with L = lens[unit] and m = keep[b]:

@@ -221,10 +221,10 @@ reco_status reco_check(cudaStream_t stream)
     if (h) {
         if ((e = cudaMemsetAsync(p, 0, sizeof h, stream)) != cudaSuccess) return cuda_fail(e, "clear error word");
         if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
-        return fail(RECO_EDEVICE, "device error word 0x%x:%s%s%s%s%s%s", h, (h & reco::ERR_LEN) ? " length-out-of-range" : "",
+        return fail(RECO_EDEVICE, "device error word 0x%x:%s%s%s%s%s%s%s", h, (h & reco::ERR_LEN) ? " length-out-of-range" : "",
                     (h & reco::ERR_KEEP) ? " keep-out-of-range" : "", (h & reco::ERR_ID) ? " id-out-of-range" : "",
                     (h & reco::ERR_TOKEN) ? " token-out-of-range" : "", (h & reco::ERR_ROOM) ? " no-room-to-append" : "",
-                    (h & reco::ERR_INTERNAL) ? " internal-check" : "");
+                    (h & reco::ERR_INTERNAL) ? " internal-check" : "", (h & reco::ERR_NORM) ? " normaliser-not-finite" : "");
     }
     return RECO_OK;
 }
@@ -251,6 +251,32 @@ reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t
     if ((st = error_word(&err)) != RECO_OK) return st;
     cudaError_t e = reco::launch_score(*kv, q_win, lens, keep, w, pool_kernel, scale, scores, lay, err, stream);
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_score_cache launch");
+}
+
+reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int32_t *lens, const int32_t *keep,
+                                 const float *row_lse, int w, int pool_kernel, float scale, float *scores, void *ws,
+                                 size_t ws_bytes, cudaStream_t stream)
+{
+    reco_status st = check_kv(kv);
+    if (st != RECO_OK) return st;
+    if (!q_win || !lens || !row_lse || !scores) return fail(RECO_EINVAL, "NULL q_win, lens, row_lse or scores");
+    if (!al16(q_win) || ((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u) || ((uintptr_t)keep & 3u) ||
+        ((uintptr_t)row_lse & 3u))
+        return fail(RECO_EINVAL, "q_win must be 16-byte aligned, lens, keep, row_lse and scores 4-byte aligned");
+    if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
+    if (pool_kernel < 1 || (pool_kernel & 1) == 0) return fail(RECO_EINVAL, "pool_kernel %d must be odd and >= 1", pool_kernel);
+    if (!(scale == scale)) return fail(RECO_EINVAL, "scale is NaN");
+    const int G = kv->H_q / kv->H_kv;
+    if ((long long)G * w > 4096) return fail(RECO_EUNSUPPORTED, "G*w = %lld window rows exceed 4096", (long long)G * w);
+    if (!reco::score_shape_supported(*kv, w))
+        return fail(RECO_EUNSUPPORTED, "G*w*d too large for the scoring kernels (G %d, w %d, d %d)", G, w, kv->d);
+    reco::ScoreWs lay = reco::score_ws_layout(*kv, w, ws);
+    if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_score_lse(*kv, q_win, lens, keep, row_lse, w, pool_kernel, scale, scores, lay, err,
+                                           stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_score_cache_lse launch");
 }
 
 reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t *lens, const int32_t *keep, int w,

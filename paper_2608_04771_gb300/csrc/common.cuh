@@ -14,6 +14,7 @@ enum : unsigned {
     ERR_TOKEN = 8u,  // an answer token outside [0, V)
     ERR_ROOM = 16u,  // no room to append a decoded row
     ERR_INTERNAL = 32u,  // an internal consistency check failed (the access was skipped)
+    ERR_NORM = 64u,  // a window row's log-normaliser passed to scoring is not finite
 };
 
 constexpr float kLog2e = 1.4426950408889634f;

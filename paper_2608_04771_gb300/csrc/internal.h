@@ -66,6 +66,9 @@ DecodeWs decode_ws_layout(const reco_kv &kv, void *base);
 // Launchers return cudaSuccess or the launch error.  All arguments validated by the caller.
 cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
                          int pool, float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s);
+cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep,
+                             const float *row_lse, int w, int pool, float scale, float *scores, const ScoreWs &ws,
+                             unsigned *err, cudaStream_t s);
 cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
                                   const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
                                   unsigned *err, cudaStream_t s);

@@ -131,6 +131,34 @@ __global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, 
     rowb[i] = m + log2f(z);
 }
 
+// Row normalisers from log-sum-exps the decode already produced (Eq. 2 with one pass over
+// K).  Window row (g, t) is query head g of the token at position L - w + t; when that
+// token was decoded the cache held exactly the keys j <= L - w + t that Eq. 2's causal
+// mask gives the row, so the decode's natural-log normaliser lse of that query head is
+// the row's: b_r = lse * log2(e).  row_lse is [w][rows_q] (rows_q = layers * B * H_q,
+// query heads in q order).  A non-finite normaliser raises ERR_NORM and leaves the row's
+// normaliser at +inf, so the row adds nothing to the scores.
+__global__ void score_rowb_from_lse(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap, int R, int G,
+                                    int Hq, int Hkv, long rows_q, const float *__restrict__ row_lse,
+                                    float *__restrict__ rowb, long units, unsigned *err)
+{
+    const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= units * R) return;
+    const long u = i / R;
+    const int r = (int)(i % R);
+    const int L = lens[u];
+    if (L < w || L > L_cap || mask.skip(u, L, w, L_cap)) return;
+    const int g = r / w, t = r % w;
+    const long qi = (u / Hkv) * Hq + (u % Hkv) * G + g;
+    const float lse = row_lse[(long)t * rows_q + qi];
+    if (!isfinite(lse)) {
+        raise_error(err, ERR_NORM);
+        rowb[i] = INFINITY;
+        return;
+    }
+    rowb[i] = lse * kLog2e;
+}
+
 // Pass 2: one thread per candidate key, its key row held in registers; the window
 // queries sit in shared memory and are read by broadcast.
 template <typename T, int D>
@@ -234,24 +262,27 @@ cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const in
                                   float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
 bool score_tc_supported(const reco_kv &kv, int w);
 
+// SIMT passes; with pass1 false the row normalisers are already in ws.rowb.
 template <typename T, int D>
 static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *lens, ScoreMask mask, int w,
-                              float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s)
+                              float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool pass1 = true)
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     const int G = kv.H_q / kv.H_kv, R = G * w;
     const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
     const T *K = (const T *)kv.k;
-    int bx = R < 256 ? ((R + 31) / 32) * 32 : 256;
-    dim3 g1(nch, (unsigned)units, (R + bx - 1) / bx);
-    score_rowstats_simt<T, D><<<g1, bx, 0, s>>>(q_win, K, lens, mask, w, G, kv.H_q, kv.H_kv, kv.L_cap, R,
-                                                nch, c2, ws.part_m, ws.part_z, err);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    long n = units * R;
-    score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch, ws.part_m,
-                                                              ws.part_z, ws.rowb, units);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
+    if (pass1) {
+        int bx = R < 256 ? ((R + 31) / 32) * 32 : 256;
+        dim3 g1(nch, (unsigned)units, (R + bx - 1) / bx);
+        score_rowstats_simt<T, D><<<g1, bx, 0, s>>>(q_win, K, lens, mask, w, G, kv.H_q, kv.H_kv, kv.L_cap, R,
+                                                    nch, c2, ws.part_m, ws.part_z, err);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        long n = units * R;
+        score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch, ws.part_m,
+                                                                  ws.part_z, ws.rowb, units);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     size_t smem = ((size_t)R * D + R) * sizeof(float);
     e = cudaFuncSetAttribute(score_colsum_simt<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
@@ -269,6 +300,18 @@ bool score_shape_supported(const reco_kv &kv, int w)
     size_t R = (size_t)(kv.H_q / kv.H_kv) * w;
     if (score_tc_supported(kv, w)) return true;
     return (kv.d == 64 || kv.d == 128) && (R * kv.d + R) <= kSimtMaxQ;
+}
+
+static cudaError_t score_simt_any(const reco_kv &kv, const void *q_win, const int32_t *lens, ScoreMask mask, int w,
+                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool pass1)
+{
+    if (kv.dtype == RECO_F32)
+        return kv.d == 64 ? score_simt<float, 64>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s, pass1)
+                          : score_simt<float, 128>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s, pass1);
+    return kv.d == 64
+               ? score_simt<__nv_bfloat16, 64>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws, err, s, pass1)
+               : score_simt<__nv_bfloat16, 128>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws, err, s,
+                                                pass1);
 }
 
 cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
@@ -300,14 +343,40 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
         }
     }
     if (!used_tc) {
-        if (kv.dtype == RECO_F32)
-            e = kv.d == 64 ? score_simt<float, 64>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s)
-                           : score_simt<float, 128>(kv, (const float *)q_win, lens, mask, w, c2, ws, err, s);
-        else
-            e = kv.d == 64
-                    ? score_simt<__nv_bfloat16, 64>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws, err, s)
-                    : score_simt<__nv_bfloat16, 128>(kv, (const __nv_bfloat16 *)q_win, lens, mask, w, c2, ws,
-                                                     err, s);
+        e = score_simt_any(kv, q_win, lens, mask, w, c2, ws, err, s, true);
+        if (e != cudaSuccess) return e;
+    }
+    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,
+                                                                            pool, scores);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep,
+                             const float *row_lse, int w, int pool, float scale, float *scores, const ScoreWs &ws,
+                             unsigned *err, cudaStream_t s)
+{
+    const float c2 = scale * kLog2e;
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const ScoreMask mask{keep, kv.B, kv.H_kv};
+    const int G = kv.H_q / kv.H_kv, R = G * w;
+    const long rows_q = (long)kv.n_layers * kv.B * kv.H_q;
+    const bool tc = kv.dtype == RECO_BF16 && score_tc_supported(kv, w);
+    cudaError_t e;
+    if (tc && keep) {
+        score_unit_list<<<1, 1024, 0, s>>>(lens, mask, w, kv.L_cap, (int)units, ws.ulist, ws.ucount);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    score_rowb_from_lse<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, G, kv.H_q,
+                                                                           kv.H_kv, rows_q, row_lse, ws.rowb, units,
+                                                                           err);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    bool used = false;
+    if (tc) {
+        e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used);
+        if (e != cudaSuccess) return e;
+    }
+    if (!used) {
+        e = score_simt_any(kv, q_win, lens, mask, w, c2, ws, err, s, false);
         if (e != cudaSuccess) return e;
     }
     score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,

@@ -20,7 +20,7 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = ran
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
+           "reco_score_cache_lse", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
            "reco_answer_ppl", "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
 
@@ -63,6 +63,7 @@ def lib():
     L.reco_last_error.restype = ctypes.c_char_p
     L.reco_check.argtypes = [vp]
     L.reco_score_cache.argtypes = [kvp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
+    L.reco_score_cache_lse.argtypes = [kvp, vp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
@@ -70,8 +71,8 @@ def lib():
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
     L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
-                 "reco_score_cache", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty",
-                 "reco_penalty_sample", "reco_answer_ppl", "reco_answer_ppl_static"):
+                 "reco_score_cache", "reco_score_cache_lse", "reco_select_compact", "reco_decode_attn",
+                 "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl", "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
     _lib = L
     return L
@@ -161,6 +162,15 @@ def reco_score_cache(kv: reco_kv, q_win, lens, w: int, pool_kernel: int, scale: 
     """keep (optional [B] int32): skip the units of sequences with keep[b] >= lens."""
     _ok(lib().reco_score_cache(ctypes.byref(kv), _ptr(q_win), _ptr(lens), _ptr(keep), int(w), int(pool_kernel),
                                float(scale), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_score_cache_lse(kv: reco_kv, q_win, lens, row_lse, w: int, pool_kernel: int, scale: float, scores, ws,
+                         keep=None, stream=None):
+    """Eq. 2 with the window rows' normalisers from the decode: row_lse [w, Ly, B, Hq]
+    float32 holds the lse reco_decode_attn returned for each window token's query."""
+    _ok(lib().reco_score_cache_lse(ctypes.byref(kv), _ptr(q_win), _ptr(lens), _ptr(keep), _ptr(row_lse), int(w),
+                                   int(pool_kernel), float(scale), _ptr(scores), _ptr(ws), ws.numel(),
+                                   _stream(stream)))
 
 
 def reco_select_compact(kv: reco_kv, scores, lens, keep, w: int, kept_idx, ws, stream=None):

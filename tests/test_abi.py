@@ -116,6 +116,15 @@ def test_device_calls_validate_before_launch(L):
     assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
     st = L.reco_score_cache(ctypes.byref(_kv(k=17)), vp(16), vp(16), None, 16, 7, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    # the lse form of Eq. 2 checks its row normalisers on top of reco_score_cache's checks
+    st = L.reco_score_cache_lse(ctypes.byref(kv), vp(16), vp(16), None, None, 16, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"row_lse" in L.reco_last_error()
+    st = L.reco_score_cache_lse(ctypes.byref(kv), vp(16), vp(16), None, vp(18), 16, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    st = L.reco_score_cache_lse(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 0, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
+    st = L.reco_score_cache_lse(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
     st = L.reco_select_compact(ctypes.byref(kv), None, vp(16), vp(16), 16, None, ws, 10, None)
     assert st == reco.RECO_EINVAL
     st = L.reco_decode_attn(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 0.1, vp(16), 0, None, ws, 10, None)

@@ -1,0 +1,157 @@
+"""reco_score_cache_lse: Eq. 2 with the window rows' normalisers taken from the decode.
+
+The window queries are decoded one token at a time (each call appends the token's key and
+value and returns the log-sum-exp of its query over the keys it sees), then the scores of
+the final cache come from one pass over K with those log-sum-exps.  They are compared with
+the oracle's Eq. 2 scores of the same cache and window (float64, its own normalisers),
+element by element, and the kept sets with the oracle's selection."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import assert_kept_match, assert_scores_close, gpu_select, np32
+from paper_2608_04771_gb300 import reco
+from paper_2608_04771_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2608_04771_gb300 import build
+    build.build()
+    reco.lib()
+
+
+def _window_case(wl, L_final):
+    """Full cache, window queries, and the per-unit initial lengths L_final - w."""
+    Kf, Vf = W.make_cache(wl, DEV, canary=False)
+    q_win = W.make_qwin(wl, DEV)
+    lens_f = np.asarray(L_final, np.int32)
+    return Kf, Vf, q_win, lens_f, lens_f - wl.w
+
+
+def _rows_at(X, pos):
+    """X[l, b, h, pos[l, b, h], :] for every unit."""
+    idx = torch.from_numpy(pos.astype(np.int64)).to(DEV)[..., None, None].expand(*pos.shape, 1, X.shape[-1])
+    return torch.gather(X, 3, idx).squeeze(3).contiguous()
+
+
+def _decode_window(wl, Kf, Vf, q_win, lens0):
+    """Decode the w window tokens into a cache that starts at lens0 rows: returns the cache,
+    the final lengths (device) and row_lse [w, Ly, B, Hq] from the decode calls."""
+    K = Kf.clone()
+    V = Vf.clone()
+    kv = reco.make_kv(K, V, wl.h_q)
+    ws = reco.workspace(reco.RECO_OP_DECODE, kv, 0, DEV)
+    lens = torch.from_numpy(lens0.copy()).to(DEV)
+    row_lse = torch.empty((wl.w, wl.layers, wl.batch, wl.h_q), dtype=torch.float32, device=DEV)
+    out = torch.empty((wl.layers, wl.batch, wl.h_q, wl.d), dtype=torch.float32, device=DEV)
+    for t in range(wl.w):
+        kn, vn = _rows_at(Kf, lens0 + t), _rows_at(Vf, lens0 + t)
+        q = q_win[:, :, :, t, :].contiguous()
+        reco.reco_decode_attn(kv, q, kn, vn, lens, wl.scale(), out, row_lse[t], ws)
+    reco.reco_check()
+    return K, V, lens, row_lse
+
+
+def _score_lse(wl, K, V, q_win, lens, row_lse, keep=None, fill=0.0):
+    kv = reco.make_kv(K, V, wl.h_q)
+    scores = torch.full(K.shape[:4], fill, dtype=torch.float32, device=DEV)
+    ws = reco.workspace(reco.RECO_OP_SCORE, kv, wl.w, DEV)
+    reco.reco_score_cache_lse(kv, q_win, lens, row_lse, wl.w, wl.pool, wl.scale(), scores, ws, keep=keep)
+    return scores
+
+
+def _compare(wl, got, ora, lens_f, skip=()):
+    for l in range(wl.layers):
+        for b in range(wl.batch):
+            if b in skip:
+                continue
+            for h in range(wl.h_kv):
+                nc = int(lens_f[l, b, h]) - wl.w
+                assert_scores_close(got[l, b, h, :nc], ora[l, b, h, :nc], f"unit {(l, b, h)}")
+
+
+CASES = [
+    # (workload, reduction): bf16 on the tensor-core pass, fp32 and d 64 on the SIMT pass
+    ("7b", dict(layers=2, batch=2, L=900, decode_steps=40)),
+    ("32b", dict(layers=1, batch=2, L=700, decode_steps=70)),
+    ("7b", dict(layers=1, batch=2, h_q=8, h_kv=2, d=64, L=600, decode_steps=40, w=24)),
+    ("tiny", dict(L=512, decode_steps=20)),
+]
+
+
+@pytest.mark.parametrize("name,red", CASES)
+def test_lse_scores_from_decoded_window(name, red):
+    """The normalisers come from the library's own decode of the window tokens."""
+    wl = W.WORKLOADS[name].reduced(**red)
+    rng = np.random.default_rng(11)
+    L_final = rng.integers(wl.w + 1, wl.L_cap - 2, (wl.layers, wl.batch, wl.h_kv)).astype(np.int32)
+    L_final[0, 0, 0] = wl.w  # no candidates at all
+    Kf, Vf, q_win, lens_f, lens0 = _window_case(wl, L_final)
+    K, V, lens, row_lse = _decode_window(wl, Kf, Vf, q_win, lens0)
+    assert np.array_equal(lens.cpu().numpy(), lens_f)
+    got = _score_lse(wl, K, V, q_win, lens, row_lse).cpu().numpy()
+    reco.reco_check()
+    ora = oracle.score_cache(np32(q_win), np32(Kf), lens_f, wl.w, wl.pool, wl.scale())
+    _compare(wl, got, ora, lens_f)
+
+
+def test_lse_scores_from_oracle_normalisers():
+    """The normalisers come from the oracle's decode of each window row (fp64 rounded to
+    fp32), so this isolates the one-pass scoring from the decode."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=2, L=1300, decode_steps=40)
+    L_final = np.random.default_rng(3).integers(wl.w + 1, wl.L_cap, (2, 2, wl.h_kv)).astype(np.int32)
+    Kf, Vf, q_win, lens_f, lens0 = _window_case(wl, L_final)
+    qn, Kn, Vn = np32(q_win), np32(Kf), np32(Vf)
+    row_lse = np.stack([oracle.decode_batch(qn[:, :, :, t, :], Kn, Vn, lens0 + t + 1, wl.scale())[1]
+                        for t in range(wl.w)]).astype(np.float32)
+    lens = torch.from_numpy(lens_f).to(DEV)
+    got = _score_lse(wl, Kf, Vf, q_win, lens, torch.from_numpy(row_lse).to(DEV)).cpu().numpy()
+    reco.reco_check()
+    ora = oracle.score_cache(qn, Kn, lens_f, wl.w, wl.pool, wl.scale())
+    _compare(wl, got, ora, lens_f)
+
+
+def test_lse_keep_mask_and_selection():
+    """With keep counts, only the sequences compressed now are scored (the others' rows of
+    scores stay as they were), and the kept sets match the oracle's selection up to the
+    tie band."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=3, L=1500, decode_steps=40)
+    L_final = np.random.default_rng(8).integers(800, wl.L_cap, (2, 3, wl.h_kv)).astype(np.int32)
+    L_final[:, 1, :] = 1200  # one length for the whole sequence: its keep count below is a no-op
+    Kf, Vf, q_win, lens_f, lens0 = _window_case(wl, L_final)
+    K, V, lens, row_lse = _decode_window(wl, Kf, Vf, q_win, lens0)
+    keep = np.array([400, 1200, 700], np.int32)  # sequence 1 keeps its whole cache: skipped
+    keep_t = torch.from_numpy(keep).to(DEV)
+    scores = _score_lse(wl, K, V, q_win, lens, row_lse, keep=keep_t, fill=-7.0)
+    got = scores.cpu().numpy()
+    reco.reco_check()
+    assert np.all(got[:, 1] == -7.0)
+    ora = oracle.score_cache(np32(q_win), np32(Kf), lens_f, wl.w, wl.pool, wl.scale())
+    _compare(wl, got, ora, lens_f, skip=(1,))
+    kept = gpu_select(wl, K, V, scores, lens, keep).cpu().numpy()
+    reco.reco_check()
+    for l in range(wl.layers):
+        for b in (0, 2):
+            for h in range(wl.h_kv):
+                L = int(lens_f[l, b, h])
+                m = min(int(keep[b]), L)
+                ora_idx = oracle.select_unit(ora[l, b, h].astype(np.float32), L, wl.w, m)
+                assert_kept_match(kept[l, b, h], ora_idx, ora[l, b, h], L, wl.w, m, f"unit {(l, b, h)}")
+
+
+def test_non_finite_normaliser_sets_device_error():
+    wl = W.WORKLOADS["7b"].reduced(layers=1, batch=1, L=300, decode_steps=4)
+    Kf, Vf, q_win, lens_f, _ = _window_case(wl, np.full((1, 1, wl.h_kv), 300, np.int32))
+    row_lse = torch.full((wl.w, 1, 1, wl.h_q), 5.0, dtype=torch.float32, device=DEV)
+    row_lse[3, 0, 0, 2] = float("nan")
+    scores = _score_lse(wl, Kf, Vf, q_win, torch.from_numpy(lens_f).to(DEV), row_lse)
+    with pytest.raises(reco.RecoError) as e:
+        reco.reco_check()
+    assert e.value.status == reco.RECO_EDEVICE and "normaliser" in str(e.value)
+    assert torch.isfinite(scores).all()
+    reco.reco_check()
