@@ -580,10 +580,14 @@ def run_trace(args):
                                f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
                                f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
                    "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically",
-                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty and draw)"
-                   if use_graph else "direct calls"},
+                   "window": "Eq. 2's window queries are the last w decoded tokens' queries; a boundary scores "
+                             "in one pass with their decode lse (kept in a device ring) when none of the "
+                             "compressing sequences was compressed within the window, else in two passes",
+                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty and draw "
+                                       "+ lse ring push)" if use_graph else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),
+                  "boundary_scorings": {"one_pass_decode_lse": ev.lse_scorings, "two_pass": ev.two_pass_scorings},
                   "stops": sum(1 for p in ev.probes if p[2]),
                   "peak_cache_bytes": ev.peak_cache_bytes,
                   "mean_cache_bytes": ev.cache_byte_tokens / max(ev.tokens, 1),

@@ -152,6 +152,20 @@ reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int
                                  const float *row_lse, int w, int pool_kernel, float scale, float *scores, void *ws,
                                  size_t ws_bytes, cudaStream_t stream);
 
+/* Keeps the decode's log-sum-exps of the last tokens on the device for
+ * reco_score_cache_lse (Sec. 3.2's observation window): copies lse[0:n] into rows
+ * *slot and *slot + slots of ring and advances *slot to (*slot + 1) % slots, all on
+ * the device, so a captured graph can push every token.  The second half of the ring
+ * mirrors the first, so the rows of the last w <= slots pushes are one contiguous
+ * [w][n] array: ring[s0 .. s0 + w - 1] with s0 = (*slot - w) mod slots, which is
+ * reco_score_cache_lse's row_lse when lse is the decode's output for each token.
+ *   lse  : [n] float32 (device), e.g. the lse output of reco_decode_attn (n =
+ *          n_layers * B * H_q)
+ *   ring : [2 * slots][n] float32 (device, two rows written)
+ *   slot : int64 (device, read and advanced); a value outside [0, slots) writes
+ *          nothing and sets the device error word.                              */
+reco_status reco_lse_push(const float *lse, int64_t n, float *ring, int slots, int64_t *slot, cudaStream_t stream);
+
 /* Top-m selection and in-place compaction (Sec. 3.2: keep the m_i best tokens,
  * the latest w always retained; compress the L cached tokens down to m_i).
  * For unit (layer, b, h) with L = lens[unit] and m = keep[b]:

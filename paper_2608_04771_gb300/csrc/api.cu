@@ -279,6 +279,19 @@ reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_score_cache_lse launch");
 }
 
+reco_status reco_lse_push(const float *lse, int64_t n, float *ring, int slots, int64_t *slot, cudaStream_t stream)
+{
+    if (n < 1 || slots < 1) return fail(RECO_EINVAL, "need n >= 1 and slots >= 1");
+    if (!lse || !ring || !slot) return fail(RECO_EINVAL, "NULL lse, ring or slot");
+    if (((uintptr_t)lse & 3u) || ((uintptr_t)ring & 3u) || ((uintptr_t)slot & 7u))
+        return fail(RECO_EINVAL, "lse and ring must be 4-byte aligned, slot 8-byte aligned");
+    unsigned *err;
+    reco_status st = error_word(&err);
+    if (st != RECO_OK) return st;
+    cudaError_t e = reco::launch_lse_push(lse, (long)n, ring, slots, reinterpret_cast<long long *>(slot), err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_lse_push launch");
+}
+
 reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t *lens, const int32_t *keep, int w,
                                 int32_t *kept_idx, void *ws, size_t ws_bytes, cudaStream_t stream)
 {

@@ -159,6 +159,67 @@ __global__ void score_rowb_from_lse(const int32_t *__restrict__ lens, ScoreMask 
     rowb[i] = lse * kLog2e;
 }
 
+// lse ring of 2 * slots rows: rows *slot and *slot + slots both get lse[0:n] (the second
+// half mirrors the first, so the rows of any `slots` consecutive pushes are contiguous),
+// then *slot = (*slot + 1) % slots.  One block: every thread reads the slot before thread
+// 0 advances it.
+__global__ void __launch_bounds__(1024) lse_push_kernel(const float *__restrict__ lse, long n, float *__restrict__ ring,
+                                                        int slots, long long *slot, unsigned *err)
+{
+    wait_prior_grid();  // lse (and the slot) may come from the previous kernels
+    __shared__ long long s0;
+    if (threadIdx.x == 0) s0 = *slot;
+    __syncthreads();
+    const long long s = s0;
+    if (s < 0 || s >= slots) {
+        if (threadIdx.x == 0) raise_error(err, ERR_INTERNAL);
+        return;
+    }
+    float *dst = ring + s * n, *mir = ring + (s + slots) * n;
+    // four independent loads in flight per thread before their stores
+    constexpr int U = 4;
+    if (n % 4 == 0 &&
+        ((reinterpret_cast<uintptr_t>(lse) | reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(mir)) & 15u) == 0) {
+        const float4 *src4 = reinterpret_cast<const float4 *>(lse);
+        float4 *dst4 = reinterpret_cast<float4 *>(dst), *mir4 = reinterpret_cast<float4 *>(mir);
+        const long n4 = n / 4;
+        for (long i0 = threadIdx.x; i0 < n4; i0 += (long)U * blockDim.x) {
+            float4 v[U];
+#pragma unroll
+            for (int k = 0; k < U; ++k) {
+                const long i = i0 + (long)k * blockDim.x;
+                if (i < n4) v[k] = src4[i];
+            }
+#pragma unroll
+            for (int k = 0; k < U; ++k) {
+                const long i = i0 + (long)k * blockDim.x;
+                if (i < n4) {
+                    dst4[i] = v[k];
+                    mir4[i] = v[k];
+                }
+            }
+        }
+    } else {
+        for (long i0 = threadIdx.x; i0 < n; i0 += (long)U * blockDim.x) {
+            float v[U];
+#pragma unroll
+            for (int k = 0; k < U; ++k) {
+                const long i = i0 + (long)k * blockDim.x;
+                if (i < n) v[k] = lse[i];
+            }
+#pragma unroll
+            for (int k = 0; k < U; ++k) {
+                const long i = i0 + (long)k * blockDim.x;
+                if (i < n) {
+                    dst[i] = v[k];
+                    mir[i] = v[k];
+                }
+            }
+        }
+    }
+    if (threadIdx.x == 0) *slot = (s + 1) % slots;
+}
+
 // Pass 2: one thread per candidate key, its key row held in registers; the window
 // queries sit in shared memory and are read by broadcast.
 template <typename T, int D>
@@ -349,6 +410,13 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
     score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,
                                                                             pool, scores);
     return cudaGetLastError();
+}
+
+cudaError_t launch_lse_push(const float *lse, long n, float *ring, int slots, long long *slot, unsigned *err,
+                            cudaStream_t s)
+{
+    cudaError_t e = launch_pdl(lse_push_kernel, dim3(1), dim3(1024), 0, s, lse, n, ring, slots, slot, err);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep,

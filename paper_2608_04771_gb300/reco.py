@@ -20,7 +20,7 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = ran
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_score_cache_lse", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
+           "reco_score_cache_lse", "reco_lse_push", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
            "reco_answer_ppl", "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
 
@@ -64,6 +64,7 @@ def lib():
     L.reco_check.argtypes = [vp]
     L.reco_score_cache.argtypes = [kvp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_score_cache_lse.argtypes = [kvp, vp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
+    L.reco_lse_push.argtypes = [vp, ctypes.c_int64, vp, i32, vp, vp]
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
@@ -71,8 +72,9 @@ def lib():
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
     L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
-                 "reco_score_cache", "reco_score_cache_lse", "reco_select_compact", "reco_decode_attn",
-                 "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl", "reco_answer_ppl_static"):
+                 "reco_score_cache", "reco_score_cache_lse", "reco_lse_push", "reco_select_compact",
+                 "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
+                 "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
     _lib = L
     return L
@@ -162,6 +164,16 @@ def reco_score_cache(kv: reco_kv, q_win, lens, w: int, pool_kernel: int, scale: 
     """keep (optional [B] int32): skip the units of sequences with keep[b] >= lens."""
     _ok(lib().reco_score_cache(ctypes.byref(kv), _ptr(q_win), _ptr(lens), _ptr(keep), int(w), int(pool_kernel),
                                float(scale), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_lse_push(lse, ring, slot, stream=None):
+    """ring[slot] = ring[slot + S] = lse (flattened); slot = (slot + 1) % S, on the device.
+    ring [2 * S, n] float32 (the second half mirrors the first), slot a one-element int64
+    device tensor."""
+    n = lse.numel()
+    if ring.dim() < 2 or ring[0].numel() != n or ring.shape[0] % 2:
+        raise ValueError("ring must have an even number of rows of lse.numel() floats")
+    _ok(lib().reco_lse_push(_ptr(lse), n, _ptr(ring), int(ring.shape[0]) // 2, _ptr(slot), _stream(stream)))
 
 
 def reco_score_cache_lse(kv: reco_kv, q_win, lens, row_lse, w: int, pool_kernel: int, scale: float, scores, ws,

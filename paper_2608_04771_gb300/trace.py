@@ -121,6 +121,8 @@ class TraceEvents:
     compressions: int = 0      # per-sequence compressions
     peak_cache_bytes: int = 0  # max over tokens of the K+V bytes held by the active sequences
     cache_byte_tokens: float = 0.0  # sum over tokens of the K+V bytes held (for the mean)
+    lse_scorings: int = 0      # boundary scorings in one pass, normalisers from the decode
+    two_pass_scorings: int = 0  # boundary scorings in two passes (a window not all decoded since)
 
 
 class Trace:
@@ -155,7 +157,7 @@ class Trace:
         self.step_idx = [0] * spec.batch
         self.out_dtype = out_dtype
         self.ids = torch.from_numpy(W.make_reflection_ids(wl)).to(device) if wl.vocab else None
-        self.staging = _Staging(2 * spec.batch, device)
+        self.staging = _Staging(3 * spec.batch + wl.w, device)
         self._pool = None
         self._answers = {}
         if input_pool:
@@ -164,7 +166,6 @@ class Trace:
             self._pool = (torch.stack([x[0] for x in ins]), torch.stack([x[1] for x in ins]),
                           torch.stack([x[2] for x in ins]),
                           torch.stack([self._token_logits(t) for t in range(input_pool)]) if wl.vocab else None,
-                          torch.stack([self._window_queries(t) for t in range(8)]),
                           torch.stack([self._token_draws(t) for t in range(input_pool)]) if wl.vocab else None)
             del ins
             # the answers of every probe the rewards can trigger, drawn before the loop runs
@@ -174,15 +175,26 @@ class Trace:
                     t = int(self.ends[sq][k])
                     if t < spec.generated and r[k - 1] >= np.float32(wl.tau_h) and r[k] >= np.float32(wl.tau_h):
                         self._answers[(t, sq)] = self._answer(t, sq)
+        # The decode's lse of the last R tokens (ring row t % R holds token t's, mirrored in
+        # row t % R + R so that any w consecutive tokens are contiguous rows; with an input
+        # pool R is its size, so one device counter selects both) and, per active
+        # sequence, how many tokens were decoded since its last compression: Eq. 2's window
+        # rows are those tokens' queries, and their lse are the rows' normalisers while the
+        # cache has not been compressed since they were decoded.
+        self.R = input_pool if input_pool else 64
+        if self.R < wl.w:
+            raise ValueError(f"input_pool {input_pool} is shorter than the window {wl.w}")
+        self.lse_ring = torch.zeros((2 * self.R, wl.layers, spec.batch, wl.h_q), dtype=torch.float32,
+                                    device=device)
+        self.slot_dev = torch.zeros(1, dtype=torch.long, device=device)
+        self._side = torch.cuda.Stream(device=device) if use_graph else None  # graph branch of the ring push
+        self._slot_t = -1  # the token whose ring slot slot_dev holds
+        self.since = [0] * spec.batch
         self._rebuild()
 
     # ---------------------------------------------------------------- inputs
     def _token_inputs(self, t: int):
         return W.make_decode_step(self.wl, 1000 + t, self.device)
-
-    def _window_queries(self, t: int):
-        wl = self.wl
-        return W.randn((wl.layers, wl.batch, wl.h_q, wl.w, wl.d), wl, 5_000_000 + t, self.device)
 
     def _token_logits(self, t: int):
         return W.randn((self.wl.batch, self.wl.vocab), self.wl, 9_000_000 + t, self.device, torch.float32) * 2.0
@@ -194,9 +206,6 @@ class Trace:
             return self._pool[0][i], self._pool[1][i], self._pool[2][i]
         return self._token_inputs(t)
 
-    def window_queries(self, t: int):
-        return self._pool[4][t % 8] if self._pool else self._window_queries(t)
-
     def token_logits(self, t: int):
         return self._pool[3][t % self.input_pool].clone() if self._pool else self._token_logits(t)
 
@@ -205,7 +214,7 @@ class Trace:
 
     def token_draws(self, t: int):
         """[B] uniform draws of token t's sampling step, full batch."""
-        return self._pool[5][t % self.input_pool] if self._pool else self._token_draws(t)
+        return self._pool[4][t % self.input_pool] if self._pool else self._token_draws(t)
 
     def answer(self, t: int, seq: int):
         """Answer logits / tokens of a probe of sequence `seq` at token t (confident on even probes)."""
@@ -244,10 +253,20 @@ class Trace:
             return self._slot_view(t % self.input_pool, 4)
         return self._sel(self._token_draws(t), 0)
 
-    def active_window_queries(self, t: int):
+    def _window(self, toks, slots, rows):
+        """Eq. 2's window queries of the sequences at batch positions `rows`: their queries of
+        the tokens `toks` (the last w decoded; input-pool slots `slots`), written into those
+        rows of q_win [Ly, B, Hq, w, d] (the other rows are not read by a masked scoring)."""
+        # moved as 16-byte elements (a query row of d values is d * es / 16 of them)
         if self._apool is not None:
-            return self._awin[t % 8]
-        return self._sel(self._window_queries(t))
+            off, nb, dt, shape = self._slot_meta[0]
+            Q = self._apool[:, off:off + nb].view(torch.complex128).view(self.input_pool, *shape[:-1], -1)
+            qs = Q.permute(0, 2, 1, 3, 4)[slots[:, None], rows[None, :]]  # [w, k, Ly, Hq, d/8], one gather
+        else:
+            qs = torch.stack([self._sel(self._token_inputs(tt)[0]) for tt in toks]).permute(0, 2, 1, 3, 4)[:, rows]
+            qs = qs.contiguous().view(torch.complex128)
+        self.q_win.view(torch.complex128).permute(1, 3, 0, 2, 4)[rows] = qs.permute(1, 0, 2, 3, 4)
+        return self.q_win
 
     # ---------------------------------------------------------------- plumbing
     def _active_pool(self):
@@ -256,10 +275,9 @@ class Trace:
         laid out like the captured graph's static inputs (each part 256-byte aligned), so a
         token's inputs arrive in a single copy."""
         if not self._pool:
-            self._awin = None
             return None
         P = self.input_pool
-        Q, KN, VN, Z, WQ, U = self._pool
+        Q, KN, VN, Z, U = self._pool
         sel = (lambda x, d: x) if self._full_batch() else (lambda x, d: x.index_select(d, self.idx_dev))
         parts = [sel(Q, 2), sel(KN, 2), sel(VN, 2)] + ([] if Z is None else [sel(Z, 1), sel(U, 1)])
         self._slot_meta, cols, off = [], [], 0
@@ -271,7 +289,6 @@ class Trace:
                 cols.append(torch.zeros((P, pad), dtype=torch.uint8, device=x.device))
             self._slot_meta.append((off, nb, x.dtype, tuple(x.shape[1:])))
             off += nb + pad
-        self._awin = sel(WQ, 2).contiguous()
         return torch.cat(cols, dim=1)
 
     def _slot_view(self, i: int, k: int):
@@ -291,6 +308,7 @@ class Trace:
         self.ws_decode = reco.workspace(reco.RECO_OP_DECODE, self.kv, 0, self.device)
         self.scores = torch.zeros(self.K.shape[:4], dtype=torch.float32, device=self.device)
         self.kept = torch.zeros(self.K.shape[:4], dtype=torch.int32, device=self.device)
+        self.q_win = torch.zeros((wl.layers, self.B, wl.h_q, wl.w, wl.d), dtype=wl.torch_dtype, device=self.device)
         self.lens_dev = torch.tensor(self.lens, dtype=torch.int32, device=self.device).view(1, -1, 1).expand(
             wl.layers, -1, wl.h_kv).contiguous()
         self.ws_ppl = reco.workspace(reco.RECO_OP_PPL, None, wl.n_answer, self.device)
@@ -307,6 +325,8 @@ class Trace:
         self.lens = [self.lens[i] for i in keep_pos]
         self.full = [self.full[i] for i in keep_pos]
         self.last_comp = [self.last_comp[i] for i in keep_pos]
+        self.since = [self.since[i] for i in keep_pos]
+        self.lse_ring = self.lse_ring.index_select(2, idx).contiguous()
         self._rebuild()
 
     def _capture(self, t: int):
@@ -329,10 +349,10 @@ class Trace:
         self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
         self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
         # keep counts (row 0) and current rewards (row 1, float32 bits): one upload per boundary
-        self.g_small = torch.zeros((2, B), dtype=torch.int32, device=dev)
-        self.g_rw = self.g_small[1].view(torch.float32)
+        # keep counts | current rewards (float32 bits) | window slots and rows: one upload
+        self.g_small = torch.zeros(3 * B + wl.w, dtype=torch.int32, device=dev)
+        self.g_rw = self.g_small[B:2 * B].view(torch.float32)
         self._put_small(list(self.lens))
-        self.g_slot = torch.zeros(1, dtype=torch.long, device=dev)
         # one call outside the capture, without an append (cache and lens stay as they are)
         reco.reco_decode_attn(self.kv, self.g_q, None, None, self.lens_dev, wl.scale(), self.g_out, self.g_lse,
                               self.ws_decode)
@@ -342,23 +362,31 @@ class Trace:
             if self._apool is not None:
                 # 16-byte elements (every part is a multiple of 256 bytes): a quarter
                 # fewer nanoseconds than 8-byte ones for the same bytes
-                torch.index_select(self._apool.view(torch.complex128), 0, self.g_slot,
+                torch.index_select(self._apool.view(torch.complex128), 0, self.slot_dev,
                                    out=self.g_in.view(torch.complex128).view(1, -1))
             reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
                                   self.g_lse, self.ws_decode)
+            # the token's lse into the ring, which advances the slot (the next token's pool
+            # slot): a branch of the graph beside the penalty and draw, joined at its end
+            main = torch.cuda.current_stream()
+            fork = torch.cuda.Event()
+            fork.record(main)
+            self._side.wait_event(fork)
+            reco.reco_lse_push(self.g_lse, self.lse_ring, self.slot_dev, stream=self._side)
             if self.g_logits is not None:
                 reco.reco_penalty_sample(self.g_logits, self.ids, self.g_rw, self.g_u, self.g_tok, self.ws_sample,
                                          wl.tau_l, wl.tau_h, wl.beta)
-            if self._apool is not None:
-                self.g_slot.add_(1)
-                self.g_slot.remainder_(self.input_pool)
-        self.g_slot.fill_(t % self.input_pool if self._apool is not None else 0)
+            main.wait_stream(self._side)
+        self.slot_dev.fill_(t % self.R)
+        self._slot_t = t
         self.graph = g
 
-    def _put_small(self, keep):
-        """Upload keep counts and the active sequences' current rewards into g_small."""
+    def _put_small(self, keep, extra=()):
+        """Upload keep counts, the active sequences' current rewards and `extra` ints into
+        g_small in one copy; returns the device view written."""
         rw = np.asarray([self.current_reward(s) for s in self.active], np.float32).view(np.int32)
-        self.staging.put(np.concatenate([np.asarray(keep, np.int32), rw]), torch.int32, out=self.g_small.view(-1))
+        vals = np.concatenate([np.asarray(keep, np.int32), rw, np.asarray(extra, np.int32)])
+        return self.staging.put(vals, torch.int32, out=self.g_small[:len(vals)])
 
     def current_reward(self, s: int) -> float:
         return float(self.hist[s][-1]) if self.hist[s] else 0.0
@@ -367,6 +395,9 @@ class Trace:
     def _token(self, t: int):
         """Decode (append + attention) and penalty of token t; returns out, lse, logits."""
         wl = self.wl
+        if self._slot_t != t:  # first token after a (re)build
+            self.slot_dev.fill_(t % self.R)
+            self._slot_t = t
         if self.use_graph:
             if self.graph is None:
                 self._capture(t)
@@ -379,12 +410,15 @@ class Trace:
                     self.g_logits.copy_(self.active_logits(t))
                     self.g_u.copy_(self.active_draws(t))
             self.graph.replay()
+            self._slot_t = t + 1
             self.tokens = self.g_tok
             return self.g_out, self.g_lse, self.g_logits
         q, kn, vn = self.active_inputs(t)
         out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
         lse = torch.empty(q.shape[:3], dtype=torch.float32, device=self.device)
         reco.reco_decode_attn(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, lse, self.ws_decode)
+        reco.reco_lse_push(lse, self.lse_ring, self.slot_dev)
+        self._slot_t = t + 1
         logits = None
         if self.ids is not None:
             logits = self.active_logits(t)
@@ -405,6 +439,7 @@ class Trace:
             out, lse, logits = self._token(t)
             self.lens = [L + 1 for L in self.lens]
             self.full = [F + 1 for F in self.full]
+            self.since = [x + 1 for x in self.since]
             ev.generated += len(self.active)
             held = sum(self.lens) * row_bytes
             ev.peak_cache_bytes = max(ev.peak_cache_bytes, held)
@@ -439,19 +474,38 @@ class Trace:
                 ev.compressions += 1
             q_win = None
             if info:
-                q_win = self.active_window_queries(t)
+                comp = [self.pos[s] for s, _, _ in info]
+                # Eq. 2's window: the queries of the last w decoded tokens (ring / pool slots)
+                toks = range(t - wl.w + 1, t + 1)
+                extra = [tt % self.R for tt in toks] + comp
                 if self.use_graph and self.graph is not None:
-                    self._put_small(keep)  # keep counts and the new rewards together
-                    keep_dev = self.g_small[0]
+                    # keep counts, the new rewards and the window's slots and rows together
+                    small = self._put_small(keep, extra)
+                    keep_dev, idx = small[:self.B], small[2 * self.B:]
                 else:
-                    keep_dev = self.staging.put(keep, torch.int32)
+                    small = self.staging.put(list(keep) + extra, torch.int32)
+                    keep_dev, idx = small[:self.B], small[self.B:]
+                slots, rows = idx[:wl.w], idx[wl.w:]
+                q_win = self._window(toks, slots, rows)
                 # only the sequences compressed now are scored (keep == L skips the rest)
-                reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
-                                      self.ws_score, keep=keep_dev)
+                if all(self.since[i] >= wl.w for i in comp):
+                    # every window token was decoded on the cache as it is now, so the lse
+                    # its decode returned is its row's normaliser: one pass over K
+                    s0 = (t - wl.w + 1) % self.R
+                    reco.reco_score_cache_lse(self.kv, q_win, self.lens_dev, self.lse_ring[s0:s0 + wl.w], wl.w,
+                                              wl.pool, wl.scale(), self.scores, self.ws_score, keep=keep_dev)
+                    ev.lse_scorings += 1
+                else:
+                    reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
+                                          self.ws_score, keep=keep_dev)
+                    ev.two_pass_scorings += 1
                 reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
                                          self.ws_select)
             if on_boundary:
                 on_boundary(t, self, done, keep, q_win)
+            for i in range(len(keep)):
+                if keep[i] < self.lens[i]:
+                    self.since[i] = 0  # compressed: its earlier lse no longer match its cache
             self.lens = keep
             # early-stop probe (two consecutive top-band rewards)
             gone = set()

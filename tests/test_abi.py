@@ -125,6 +125,12 @@ def test_device_calls_validate_before_launch(L):
     assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
     st = L.reco_score_cache_lse(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 16, 7, 0.1, vp(16), ws, 10, None)
     assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    st = L.reco_lse_push(vp(16), 0, vp(16), 4, vp(16), None)
+    assert st == reco.RECO_EINVAL
+    st = L.reco_lse_push(vp(16), 10, vp(16), 4, None, None)
+    assert st == reco.RECO_EINVAL and b"NULL" in L.reco_last_error()
+    st = L.reco_lse_push(vp(16), 10, vp(16), 4, vp(20), None)
+    assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
     st = L.reco_select_compact(ctypes.byref(kv), None, vp(16), vp(16), 16, None, ws, 10, None)
     assert st == reco.RECO_EINVAL
     st = L.reco_decode_attn(ctypes.byref(kv), vp(16), vp(16), None, vp(16), 0.1, vp(16), 0, None, ws, 10, None)

@@ -155,3 +155,31 @@ def test_non_finite_normaliser_sets_device_error():
     assert e.value.status == reco.RECO_EDEVICE and "normaliser" in str(e.value)
     assert torch.isfinite(scores).all()
     reco.reco_check()
+
+
+def test_lse_push_ring_and_slot():
+    """Each push writes its ring row and the mirror row `slots` further on at the device slot
+    and advances the slot modulo `slots` (bit-exact copies), so the last w pushes are the
+    contiguous rows s0 .. s0+w-1 with s0 = (slot - w) mod slots.  An out-of-range slot
+    writes nothing and sets the error word."""
+    n, slots, w = 1000, 5, 3
+    ring = torch.full((2 * slots, n), -1.0, device=DEV)
+    slot = torch.tensor([3], dtype=torch.int64, device=DEV)
+    vals = [torch.randn(n, device=DEV) for _ in range(7)]
+    for v in vals:
+        reco.reco_lse_push(v, ring, slot)
+    reco.reco_check()
+    nxt = int(slot.item())
+    assert nxt == (3 + 7) % slots
+    assert torch.equal(ring[:slots], ring[slots:])
+    last = {(3 + i) % slots: v for i, v in enumerate(vals)}
+    for k, v in last.items():
+        assert torch.equal(ring[k], v)
+    s0 = (nxt - w) % slots
+    assert torch.equal(ring[s0:s0 + w], torch.stack(vals[-w:]))
+    slot.fill_(9)
+    before = ring.clone()
+    reco.reco_lse_push(vals[0], ring, slot)
+    with pytest.raises(reco.RecoError):
+        reco.reco_check()
+    assert torch.equal(ring, before) and int(slot.item()) == 9

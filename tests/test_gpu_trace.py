@@ -1,6 +1,8 @@
 """The step-loop trace (ragged step boundaries, compression at every boundary,
 decode between, penalty and a draw every token, answer probe on two top-band rewards,
-stopped sequences leaving the batch) replayed in lock-step by the oracle.
+stopped sequences leaving the batch) replayed in lock-step by the oracle.  Eq. 2's window
+queries are the last w decoded tokens' queries; the library scores a boundary in one pass
+from their decode lse when it can, and the oracle always from its own normalisers.
 
 The oracle keeps its own float64-computed cache state from the same seeded inputs
 (never from the GPU's results) and checks, at every token, every decode output, the
@@ -125,8 +127,8 @@ class OracleReplay:
         self.checked_boundaries += 1
 
 
-def _run(spec, track=None, decode_every=1, use_graph=False):
-    tr = trace.Trace(spec, DEV, use_graph=use_graph)
+def _run(spec, track=None, decode_every=1, use_graph=False, input_pool=0):
+    tr = trace.Trace(spec, DEV, use_graph=use_graph, input_pool=input_pool)
     rep = OracleReplay(tr, track, decode_every)
     ev = tr.run(on_token=rep.on_token, on_boundary=rep.on_boundary)
     reco.reco_check()
@@ -140,16 +142,18 @@ def _run(spec, track=None, decode_every=1, use_graph=False):
     return tr, rep, ev
 
 
-@pytest.mark.parametrize("use_graph", [False, True])
-def test_trace_reading_A_reduced(use_graph):
+@pytest.mark.parametrize("use_graph,input_pool", [(False, 0), (True, 0), (True, 64)])
+def test_trace_reading_A_reduced(use_graph, input_pool):
     # tau_h 0.6 so that this seed's Beta(2,2) rewards trigger probes (4 probes, 3 stops)
     base = W.WORKLOADS["7b"].reduced(layers=2, vocab=5000, tau_h=0.6)
     spec = trace.TraceSpec(base, batch=4, prompt=128, generated=400, step_mean=40, step_min=8, seed=4,
                            reading="A")
-    tr, rep, ev = _run(spec, use_graph=use_graph)
+    tr, rep, ev = _run(spec, use_graph=use_graph, input_pool=input_pool)
     assert rep.tie_diffs == 0  # no near-tie flips on this seed: every unit compared throughout
     assert rep.checked_tokens >= 150 and rep.checked_boundaries >= 15
     assert len(ev.probes) == 4 and sum(st for (_, _, st, _) in ev.probes) == 3
+    # steps of at least w tokens score in one pass from the decode's lse, shorter ones in two
+    assert ev.lse_scorings > 0 and ev.two_pass_scorings > 0
 
 
 def test_trace_interval_trigger():
@@ -182,3 +186,4 @@ def test_trace_full_size_sampled():
     assert rep.checked_boundaries >= 100 and rep.checked_tokens >= 100
     # near-tie flips (fp32 vs fp64 scores within 1e-5 of the cut) stop the comparison of that unit only
     assert len(rep.diverged) <= 0.05 * 2 * spec.base.layers * spec.base.h_kv, rep.diverged
+    assert ev.lse_scorings > 10 * ev.two_pass_scorings  # steps are Poisson(96)+16 >> w tokens
