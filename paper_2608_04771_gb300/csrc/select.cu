@@ -7,6 +7,9 @@
 // largest key T and how many keys equal to T are still needed; one ordered pass
 // then emits every candidate with key > T plus the first `need` with key == T in
 // index order.  The result is sorted and ties go to the lower index, with no sort.
+// select_topm_smem does the same from keys staged in shared memory (units of up to
+// kSelectSmemKeys candidates); the histogram groups equal bins of the lanes whose key
+// still matches the prefix (in the later passes, few do).
 //
 // compact_rows: one CTA per (unit, K|V, 128-byte column slice).  kept[] is strictly
 // increasing, so kept[r] >= r: the source of destination r is never a row that an
@@ -35,6 +38,9 @@ SelectWs select_ws_layout(const reco_kv &kv, void *base)
     ws.bytes = off;
     return ws;
 }
+
+// Most candidates a unit may have for the shared-memory selection (192 KB of keys).
+constexpr int kSelectSmemKeys = 48 * 1024;
 
 __device__ __forceinline__ uint32_t order_key(float f)
 {
@@ -117,8 +123,11 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
                 const uint32_t key = valid ? order_key(s[j]) : 0u;
                 const bool match = valid && (key & mask) == prefix;
                 const uint32_t bin = (key >> shift) & 255u;
-                const unsigned peers = __match_any_sync(0xffffffffu, match ? bin : 256u + lane);
-                if (match && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+                const unsigned inm = __ballot_sync(0xffffffffu, match);
+                if (match) {
+                    const unsigned peers = __match_any_sync(inm, bin);
+                    if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+                }
             }
             __syncthreads();
             if (tid < 32) {  // find the bin holding the remaining-th largest key
@@ -175,6 +184,159 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
     }
 }
 
+// The same selection with the unit's keys staged in shared memory once (all loads in
+// flight), the radix passes run from there, and the ordered emit done by warp-contiguous
+// segments: one counting sweep, one scan of the 32 warps' counts, one writing sweep.
+template <int NT>
+__global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__ scores, int32_t *lens,
+                                                       const int32_t *__restrict__ keep, int w, int B, int Hkv,
+                                                       int L_cap, int32_t *__restrict__ idx_out,
+                                                       int32_t *__restrict__ count, unsigned *err)
+{
+    static_assert(NT == 1024, "one warp per lane of the warp-count scan");
+    constexpr int NW = NT / 32;
+    extern __shared__ uint32_t keys[];  // [L - w]
+    __shared__ int hist[256];
+    __shared__ int w_gt[NW], w_eq[NW];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_remaining;
+    const long u = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int b = (int)((u / Hkv) % B);
+    const int L = lens[u], m = keep[b];
+    if (L < w || L > L_cap || m < w || m > L) {
+        if (tid == 0) {
+            count[u] = 0;
+            raise_error(err, (L < w || L > L_cap) ? ERR_LEN : ERR_KEEP);
+        }
+        return;
+    }
+    const int nc = L - w, kc = m - w;
+    const float *s = scores + u * L_cap;
+    int32_t *idx = idx_out + u * L_cap;
+    if (kc == nc) {  // keep everything: identity, nothing moves
+        for (int j = tid; j < L; j += NT) idx[j] = j;
+        if (tid == 0) count[u] = m;
+        return;
+    }
+#pragma unroll 8
+    for (int j = tid; j < nc; j += NT) keys[j] = order_key(__ldcg(s + j));
+    if (tid == 0) {
+        s_prefix = 0;
+        s_remaining = kc;
+    }
+    __syncthreads();
+    uint32_t T = 0xffffffffu;
+    int need = 0;
+    if (kc > 0) {
+        uint32_t mask = 0;
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            for (int i = tid; i < 256; i += NT) hist[i] = 0;
+            __syncthreads();
+            const uint32_t prefix = s_prefix;
+            const int remaining = s_remaining;
+            for (int jb = 0; jb < nc; jb += NT) {
+                const int j = jb + tid;
+                const bool valid = j < nc;
+                const uint32_t key = valid ? keys[j] : 0u;
+                const bool match = valid && (key & mask) == prefix;
+                const uint32_t bin = (key >> shift) & 255u;
+                // group only the lanes whose key still matches (in later passes, few do)
+                const unsigned inm = __ballot_sync(0xffffffffu, match);
+                if (match) {
+                    const unsigned peers = __match_any_sync(inm, bin);
+                    if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+                }
+            }
+            __syncthreads();
+            if (tid < 32) {  // find the bin holding the remaining-th largest key
+                int c8[8], sum = 0;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    c8[i] = hist[255 - 8 * lane - i];
+                    sum += c8[i];
+                }
+                int incl = sum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    int n = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += n;
+                }
+                int cum = incl - sum;
+                if (cum < remaining && remaining <= incl) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        if (cum + c8[i] >= remaining) {
+                            s_prefix = prefix | ((uint32_t)(255 - 8 * lane - i) << shift);
+                            s_remaining = remaining - cum;
+                            break;
+                        }
+                        cum += c8[i];
+                    }
+                }
+            }
+            mask |= 255u << shift;
+            __syncthreads();
+        }
+        T = s_prefix;
+        need = s_remaining;
+    }
+    // emit in index order: keys > T, then the first `need` keys == T
+    const int seg = (nc + NW - 1) / NW;
+    const int j0 = min(nc, wid * seg), j1 = min(nc, j0 + seg);
+    int n_gt = 0, n_eq = 0;
+    for (int jb = j0; jb < j1; jb += 32) {
+        const int j = jb + lane;
+        const uint32_t key = j < j1 ? keys[j] : 0u;
+        n_gt += __popc(__ballot_sync(0xffffffffu, j < j1 && key > T));
+        n_eq += __popc(__ballot_sync(0xffffffffu, j < j1 && key == T));
+    }
+    if (lane == 0) {
+        w_gt[wid] = n_gt;
+        w_eq[wid] = n_eq;
+    }
+    __syncthreads();
+    if (wid == 0) {  // per warp: equal keys before its segment, and output rows before it
+        const int e = w_eq[lane], g = w_gt[lane];
+        int e_inc = e;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int n = __shfl_up_sync(0xffffffffu, e_inc, o);
+            if (lane >= o) e_inc += n;
+        }
+        const int e_base = e_inc - e;
+        const int f = g + min(max(need - e_base, 0), e);
+        int f_inc = f;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int n = __shfl_up_sync(0xffffffffu, f_inc, o);
+            if (lane >= o) f_inc += n;
+        }
+        w_eq[lane] = e_base;
+        w_gt[lane] = f_inc - f;
+    }
+    __syncthreads();
+    int e_run = w_eq[wid], pos = w_gt[wid];
+    const unsigned below = (1u << lane) - 1u;
+    for (int jb = j0; jb < j1; jb += 32) {
+        const int j = jb + lane;
+        const bool valid = j < j1;
+        const uint32_t key = valid ? keys[j] : 0u;
+        const bool is_eq = valid && key == T;
+        const unsigned eb = __ballot_sync(0xffffffffu, is_eq);
+        const bool flag = (valid && key > T) || (is_eq && e_run + __popc(eb & below) < need);
+        const unsigned fb = __ballot_sync(0xffffffffu, flag);
+        if (flag) idx[pos + __popc(fb & below)] = j;
+        e_run += __popc(eb);
+        pos += __popc(fb);
+    }
+    for (int t = tid; t < w; t += NT) idx[kc + t] = nc + t;
+    if (tid == 0) {
+        count[u] = m;
+        lens[u] = m;
+    }
+}
+
 __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int32_t *__restrict__ idx_all,
                                                     const int32_t *__restrict__ count, int L_cap,
                                                     int row_bytes, unsigned *err)
@@ -219,9 +381,20 @@ cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     int32_t *idx = kept_idx ? kept_idx : ws.idx;
-    select_topm<1024><<<(unsigned)units, 1024, 0, s>>>(scores, lens, keep, w, kv.B, kv.H_kv, kv.L_cap,
-                                                       idx, ws.count, err);
-    cudaError_t e = cudaGetLastError();
+    // keys of a unit staged in shared memory when L_cap - w of them fit
+    const size_t key_bytes = (size_t)(kv.L_cap - w) * sizeof(uint32_t);
+    cudaError_t e;
+    if (key_bytes <= kSelectSmemKeys * sizeof(uint32_t)) {
+        e = cudaFuncSetAttribute(select_topm_smem<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kSelectSmemKeys * (int)sizeof(uint32_t));
+        if (e != cudaSuccess) return e;
+        select_topm_smem<1024><<<(unsigned)units, 1024, key_bytes, s>>>(scores, lens, keep, w, kv.B, kv.H_kv,
+                                                                       kv.L_cap, idx, ws.count, err);
+    } else {
+        select_topm<1024><<<(unsigned)units, 1024, 0, s>>>(scores, lens, keep, w, kv.B, kv.H_kv, kv.L_cap, idx,
+                                                           ws.count, err);
+    }
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int row_bytes = kv.d * (kv.dtype == RECO_F32 ? 4 : 2);
     dim3 grid((unsigned)units, 2, row_bytes / 128);

@@ -103,3 +103,15 @@ def test_select_bad_keep_sets_device_error_and_skips_unit():
     assert torch.equal(K[0, 0].view(torch.int16), K0[0, 0].view(torch.int16))
     assert int(lens[0, 0, 0]) == 200 and int(lens[0, 1, 0]) == 50
     reco.reco_check()  # the word was cleared and the context is still usable
+
+
+def test_select_compact_beyond_shared_memory_keys():
+    """Units with more candidates than the shared-memory selection holds (48 Ki keys) take
+    the selection that reads its keys from global memory: same results, ties included."""
+    wl = W.WORKLOADS["1.5b"].reduced(layers=1, batch=2, h_q=2, h_kv=1, L=50_000, decode_steps=8, w=32,
+                                     outliers=0)
+    assert wl.L_cap - wl.w > 48 * 1024
+    rng = np.random.default_rng(21)
+    lens = np.array([[[50_000], [49_500]]], np.int32)
+    keep = np.array([12_345, 30_001], np.int32)
+    _run_case(wl, lens, keep, _tie_scores(rng, (1, 2, 1, wl.L_cap), 4096))
