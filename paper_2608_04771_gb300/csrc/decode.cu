@@ -357,10 +357,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         return lo;
     };
-    auto snap = [&](int b) {  // a range start inside a short unit moves to the unit's start
+    auto snap = [&](int b) {  // a range start inside a short unit moves to its nearer end
         if (b >= NB) return NB;
         const int u = last_le(pb, units, b);
-        return pb[u + 1] - pb[u] <= kMaxWholeBlocks ? pb[u] : b;
+        const int ub = pb[u], ue = pb[u + 1];
+        if (ue - ub > kMaxWholeBlocks) return b;
+        return b - ub <= ue - b ? ub : ue;
     };
     // static deal interleaved across CTAs (warp wid of every CTA before warp wid+1 of
     // any): with fewer working warps than warps the work still spreads over all SMs
