@@ -264,6 +264,28 @@ def test_decode_special_cases():
     assert abs(lse - (0.25 * float(k[0].astype(np.float64) @ q.astype(np.float64)) + math.log(9))) < 1e-12
 
 
+def test_decode_lse_is_the_eq2_row_normaliser():
+    """The identity the one-pass scoring rests on, between two separate oracle functions:
+    the decode of window query t over the keys 0..L-w+t (its cache when it was decoded)
+    returns lse_t, and exp(logit - lse_t) summed over the window and averaged over the G
+    heads is Eq. 2's raw score.  A causal off-by-one or a wrong window position on either
+    side breaks it."""
+    rng = np.random.default_rng(12)
+    G, w, L, d, scale = 3, 5, 23, 8, 0.37
+    q = rng.standard_normal((G, w, d)).astype(np.float32)
+    k = rng.standard_normal((L, d)).astype(np.float32)
+    v = rng.standard_normal((L, d)).astype(np.float32)
+    raw_ref, _ = oracle.score_unit(q, k, w, scale, 1)
+    raw = np.zeros(L)
+    for g in range(G):
+        for t in range(w):
+            n = L - w + t + 1
+            _, lse = oracle.decode_unit(q[g, t], k[:n], v[:n], n, scale)
+            logits = scale * (k[:n].astype(np.float64) @ q[g, t].astype(np.float64))
+            raw[:n] += np.exp(logits - lse)
+    np.testing.assert_allclose(raw / G, raw_ref, rtol=1e-12, atol=1e-15)
+
+
 def test_decode_batch_head_grouping():
     rng = np.random.default_rng(14)
     Ly, B, Hq, Hkv, Lc, d = 2, 2, 6, 2, 12, 8
