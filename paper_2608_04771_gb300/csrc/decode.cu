@@ -330,7 +330,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // with a ring twice as deep: more bytes in flight per warp keep HBM busier once every
     // warp has many blocks; short work keeps all warps for latency.  The CTA's ring is the
     // same either way (NW * S stages).
-    const bool deep = NB >= kDeepBlocksPerWarp * total_warps;
+    // Fewer than half as many units as warps (with at least 8 blocks per warp) also
+    // takes the deep partition: there the 8-warp split would cut every unit into many
+    // pieces, whose merges cost more than the shallower rings save.
+    const bool deep =
+        NB >= kDeepBlocksPerWarp * total_warps || (NB >= 8 * total_warps && total_warps > 2 * units);
     bool aborted = false;
     {
     const int NWm = deep ? NW / 2 : NW, Sm = deep ? 2 * S : S;  // NWm * Sm == NW * S either way
