@@ -15,14 +15,19 @@ When a sequence completes a step it receives a reward v_i (Sec. 3.1), and
     keep = L, which skips their scoring and leaves them untouched;
   * if v_{i-1} >= tau_h and v_i >= tau_h, the answer probe runs (Eq. 5-6) and a
     sequence that passes PPL <= tau_p stops and leaves the batch.
+Eq. 2's observation window is the queries of the last w decoded tokens.  The lse each
+decode returns is kept in a device ring; when none of the sequences compressed at a
+boundary was compressed within its window, those lse are the window rows' normalisers
+and the scores take one pass over K (reco_score_cache_lse), else two (reco_score_cache).
 Budget base L (the paper is silent on repeated compression): reading "A" uses the
 current cache length, reading "B" the full uncompressed length so far (the keep
 count is then capped at the current length).  Lengths are tracked on the host, so
 the loop needs no device read-back except the stop flags of a probe.
 
-With use_graph, a token's decode + penalty is one captured CUDA graph over static
-input buffers (captured again whenever the batch shrinks), so the per-token host
-work is one input copy and one graph launch.
+With use_graph, a token's decode, penalty, draw and lse push are one captured CUDA
+graph over static input buffers (captured again whenever the batch shrinks), so the
+per-token host work is one graph launch (with an input pool, the graph also gathers
+the token's inputs).
 """
 from __future__ import annotations
 
@@ -348,7 +353,6 @@ class Trace:
         self.g_tok = torch.full((B,), -1, dtype=torch.int32, device=dev)
         self.g_out = torch.empty(self.g_q.shape, dtype=self.out_dtype, device=dev)
         self.g_lse = torch.empty(self.g_q.shape[:3], dtype=torch.float32, device=dev)
-        # keep counts (row 0) and current rewards (row 1, float32 bits): one upload per boundary
         # keep counts | current rewards (float32 bits) | window slots and rows: one upload
         self.g_small = torch.zeros(3 * B + wl.w, dtype=torch.int32, device=dev)
         self.g_rw = self.g_small[B:2 * B].view(torch.float32)
