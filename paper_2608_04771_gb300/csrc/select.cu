@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
                                                     int row_bytes, unsigned *err)
 {
     constexpr int P = 8;  // 16-byte pieces per 128-byte slice
-    constexpr int U = 4;  // rows per thread in flight
+    constexpr int U = 2;  // rows per thread in flight
     const long u = blockIdx.x;
     const int m = count[u];
     if (m == 0) return;
