@@ -273,8 +273,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // end to end (prefix pb) and every working warp takes one contiguous range of equal
     // length, cut across unit boundaries (a stream-K split).  A unit cut between warps
     // leaves partial (max, sum, output) triples that its last piece merges.  Short units
-    // (<= kMaxWholeBlocks blocks) are never cut: a range start inside one moves back to
-    // the unit's start, since there a merge costs more than the imbalance it removes.
+    // (<= kMaxWholeBlocks blocks) are never cut: a range start inside one moves to the
+    // unit's nearer end, since there a merge costs more than the imbalance it removes.
     int *pb = sm_pre;  // [units + 1] prefix of blocks
     const int seg = (units + blockDim.x - 1) / blockDim.x;
     const int u_lo = min(units, tid * seg), u_hi = min(units, u_lo + seg);
