@@ -74,3 +74,37 @@ def test_full_size_sampled_units(name):
         got = hp.ppl.cpu().numpy().astype(np.float64)
         assert np.all(np.abs(got - ppl_ref) <= PPL_RTOL * ppl_ref)
         assert np.array_equal(hp.stop.cpu().numpy().astype(bool), stop_ref)
+
+
+@pytest.mark.parametrize("name", ["7b", "1.5b", "32b"])
+def test_full_size_one_pass_scores_sampled(name):
+    """reco_score_cache_lse on the full workload cache, as bench.py times it: each window
+    query's normaliser is the lse of the library's decode of that query over the keys Eq. 2
+    lets it see (lens L-w+t+1, no append); sampled units against the oracle's Eq. 2 scores
+    (its own normalisers) and its selection."""
+    wl = W.WORKLOADS[name]
+    hp = driver.HotPath(wl, DEV, out_dtype=torch.float32, keep_pristine=False)
+    ws_dec = reco.workspace(reco.RECO_OP_DECODE, hp.kv, 0, DEV)
+    row_lse = torch.empty((wl.w, wl.layers, wl.batch, wl.h_q), dtype=torch.float32, device=DEV)
+    out = torch.empty((wl.layers, wl.batch, wl.h_q, wl.d), dtype=torch.float32, device=DEV)
+    for t in range(wl.w):
+        lens_t = hp.lens0 - (wl.w - 1 - t)
+        reco.reco_decode_attn(hp.kv, hp.q_win[:, :, :, t, :].contiguous(), None, None, lens_t, wl.scale(), out,
+                              row_lse[t], ws_dec)
+    scores = torch.zeros_like(hp.scores)
+    reco.reco_score_cache_lse(hp.kv, hp.q_win, hp.lens, row_lse, wl.w, wl.pool, wl.scale(), scores, hp.ws_score)
+    reco.reco_check()
+    kept = torch.full(hp.K.shape[:4], -1, dtype=torch.int32, device=DEV)
+    G = wl.G
+    units = [(0, 0, 0), (wl.layers // 2, wl.batch // 2, wl.h_kv - 1), (wl.layers - 1, wl.batch - 1, wl.h_kv // 2)]
+    saved = {u: (np32(hp.K[u[0], u[1], u[2], :wl.L]), np32(hp.q_win[u[0], u[1], u[2] * G:(u[2] + 1) * G]))
+             for u in units}
+    reco.reco_select_compact(hp.kv, scores, hp.lens, hp.keep, wl.w, kept, hp.ws_select)
+    reco.reco_check()
+    for (l, b, h) in units:
+        K0, q = saved[(l, b, h)]
+        m = int(hp.keep_host[b])
+        _, pooled = oracle.score_unit(q, K0, wl.w, wl.scale(), wl.pool)
+        assert_scores_close(scores[l, b, h, :wl.L - wl.w].cpu().numpy(), pooled, f"{name} unit {(l, b, h)}")
+        ora_idx = oracle.select_unit(pooled.astype(np.float32), wl.L, wl.w, m)
+        assert_kept_match(kept[l, b, h].cpu().numpy(), ora_idx, pooled, wl.L, wl.w, m, f"{name} unit {(l, b, h)}")
