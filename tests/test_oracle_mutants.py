@@ -53,6 +53,13 @@ MUTANTS = {
     "max-pool window one too wide": (
         "int half = pool / 2;", "int half = pool / 2 + 1;",
         [P.test_maxpool_matches_scipy]),
+    "decode lse without its max": (
+        "if (lse) *lse = mx + log(Z);", "if (lse) *lse = log(Z);",
+        [P.test_decode_lse_is_the_eq2_row_normaliser]),
+    "decode normaliser misses the last key": (
+        "for (int j = 0; j < len; ++j) Z += exp(logit[j] - mx);",
+        "for (int j = 0; j < len - 1; ++j) Z += exp(logit[j] - mx);",
+        [P.test_decode_lse_is_the_eq2_row_normaliser]),
     "decode multiplies by K instead of V": (
         "out[c] += p * (double)v[(size_t)j * d + c];", "out[c] += p * (double)k[(size_t)j * d + c];",
         [P.test_decode_matches_torch_sdpa]),
