@@ -14,7 +14,7 @@
  * OpenMP loop over independent (layer, sequence, KV-head) units in the batched
  * wrappers; each unit is computed by the same serial code.
  *
- * Readings of points the paper leaves open (each also listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - Eq. 1 with v_max == v_min (one reward, or all equal): the adjustment is 0.
  *   - Eq. 1 statistics run over all step rewards v_1..v_i, the current one included.
  *   - keep count m = clamp(floor(lambda_i * L), w, L); m counts the window.
