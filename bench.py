@@ -1,13 +1,17 @@
 """Benchmark of the ReCo hot path on GB300: compress + decode tokens/s.
 
-One step = one reasoning-step boundary of the 7B-class workload (28 layers, 28/4
-heads, d 128, bf16, batch 8, cache 16384): Eq. 1 keep counts, Eq. 2 scores,
-top-m select + in-place compaction, then 128 decode steps (append + attention over
-the ragged compacted cache, all layers per launch) each followed by the Eq. 3-4
-reflection penalty on [8, 152064] logits, and the Eq. 5-6 answer-PPL probe over
-32 answer tokens.  Tokens per step = B*L cached tokens compressed + B*128 decoded.
+One step = one reasoning-step boundary of a workload and the decode that follows.
+The default is the largest single-GPU one, the 32B-class stack (Qwen2.5-32B shape:
+64 layers, 40/8 heads, d 128, bf16, batch 4, cache 32768, window 64, Eq. 1 ratios
+spanning 0.2-0.9): Eq. 1 keep counts, Eq. 2 scores, top-m select, in-place
+compaction, then 256 decode steps (append + attention over the ragged compacted
+cache, all layers per launch).  The 7B-class workload adds the Eq. 3-4 reflection
+penalty on [8, 152064] logits after every decode step and the Eq. 5-6 answer-PPL
+probe over 32 answer tokens.  Tokens per step = B*L cached tokens compressed +
+B*steps decoded; the line also carries the two rates apart (compress_tokens_s over
+score + select + compact, decode_tokens_s over the decode launches).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 7b|1.5b|32b|tiny]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 32b|7b|1.5b|tiny|trace]
     python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
 
 Under torchrun each rank runs an independent replica (the path shards by sequence
@@ -135,21 +139,25 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def decode_traffic(dtype_tag: str):
-    """DRAM bytes per decode launch from the committed ncu summary, if it was taken
-    on the current decode kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "decode_attn_7b.md")
+def decode_traffic(wl):
+    """DRAM bytes per decode launch of this workload from the committed ncu summary
+    profiles/decode_attn_<workload>.md, if it was taken on the current decode kernel
+    source (checked by hash).  Returns (bytes or None, where the figure comes from)."""
+    name = f"decode_attn_{wl.name}.md"
+    path = os.path.join(ROOT, "profiles", name)
     if not os.path.exists(path):
-        return None
+        return None, f"none: no ncu summary profiles/{name}"
     text = open(path).read()
     m = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
     h = re.search(r"decode_source_sha256:\s*([0-9a-f]+)", text)
+    c = re.search(r"capture:\s*(.+)", text)
     if not m or not h:
-        return None
+        return None, f"none: profiles/{name} carries no per-launch DRAM bytes"
     src = open(os.path.join(ROOT, "paper_2608_04771_gb300", "csrc", "decode.cu"), "rb").read()
     if hashlib.sha256(src).hexdigest()[:16] != h.group(1)[:16]:
-        return None
-    return float(m.group(1))
+        return None, f"none: profiles/{name} was taken on another decode.cu"
+    return float(m.group(1)), (f"profile-derived, not measured in this run: profiles/{name} "
+                               f"(ncu dram__bytes_read.sum + dram__bytes_write.sum; {c.group(1).strip() if c else ''})")
 
 
 # ------------------------------------------------------------------ algorithmic work
@@ -179,85 +187,158 @@ def algorithmic(wl, keep_host):
 
 
 # ------------------------------------------------------------------ oracle timing (CPU)
-def oracle_sample(wl, units_sample: int, dec_steps_sample: int):
-    """Time the fp64 oracle on a bounded sample of the workload on the host cores and
-    extrapolate to one full step.  Returns (seconds per full step, description)."""
+class OracleSample:
+    """The fp64 oracle timed on a bounded sample of a workload on the host cores: the
+    first `units` units (whole layers of the batch, or part of layer 0) at full length
+    for score + select + compact, then `dec_steps` decode steps over them; for workloads
+    with a vocabulary, the penalty once on the full logits and the PPL on the sampled
+    sequences.  Inputs are drawn once; run() times one pass over the sample.  Nothing is
+    extrapolated inside run(): project() scales the measured pieces linearly to one full
+    step (all units, all decode steps, a penalty per decode step, the PPL of every sequence)."""
+
+    def __init__(self, wl, units: int, dec_steps: int):
+        import oracle
+        from paper_2608_04771_gb300 import workloads as W
+        oracle.build()
+        self.wl = wl
+        per_layer = wl.batch * wl.h_kv
+        if units >= per_layer:
+            Ls, Bs = min(wl.layers, -(-units // per_layer)), wl.batch
+        else:
+            Ls, Bs = 1, max(1, min(wl.batch, -(-units // wl.h_kv)))
+        self.sw = sw = wl.reduced(layers=Ls, batch=Bs)
+        K, V = W.make_cache(sw, "cpu", canary=False)
+        self.K, self.V = K.float().numpy(), V.float().numpy()
+        self.q = W.make_qwin(sw, "cpu").float().numpy()
+        self.lens = np.full((Ls, Bs, sw.h_kv), sw.L, np.int32)
+        hist = W.make_reward_history(wl)[:Bs]
+        self.keep = np.array([oracle.keep_count(oracle.retention_ratio(hist[b], wl.base, wl.delta), wl.L, wl.w)
+                              for b in range(Bs)], np.int32)
+        self.n_dec = min(dec_steps, wl.decode_steps)
+        self.dec = []
+        for s in range(self.n_dec):
+            qd, kn, vn = W.make_decode_step(sw, s, "cpu")
+            self.dec.append((qd.float().numpy(), kn.float().numpy(), vn.float().numpy()))
+        if wl.vocab:
+            self.z = W.make_vocab_logits(wl, "cpu").numpy()
+            self.ids = W.make_reflection_ids(wl)
+            self.rw = W.make_reward_history(wl)[:, -1].copy()
+            za, tok = W.make_answer(wl.reduced(batch=Bs), "cpu")
+            self.za, self.tok = za.numpy(), tok.numpy()
+
+    def run(self):
+        import oracle
+        sw, wl = self.sw, self.wl
+        t0 = time.perf_counter()
+        sc = oracle.score_cache(self.q, self.K, self.lens, sw.w, sw.pool, sw.scale())
+        idx = oracle.select_batch(sc.astype(np.float32), self.lens, self.keep, sw.w)
+        Kc, Vc = np.zeros_like(self.K), np.zeros_like(self.V)
+        for l in range(sw.layers):
+            for b in range(sw.batch):
+                m = int(self.keep[b])
+                for h in range(sw.h_kv):
+                    Kc[l, b, h, :m] = oracle.gather_unit(self.K[l, b, h], idx[l, b, h, :m])
+                    Vc[l, b, h, :m] = oracle.gather_unit(self.V[l, b, h], idx[l, b, h, :m])
+        t_comp = time.perf_counter() - t0
+        lens_c = np.broadcast_to(self.keep.reshape(1, -1, 1), self.lens.shape).copy()
+        t0 = time.perf_counter()
+        for qd, kn, vn in self.dec:
+            for l in range(sw.layers):
+                for b in range(sw.batch):
+                    for h in range(sw.h_kv):
+                        Lc = lens_c[l, b, h]
+                        Kc[l, b, h, Lc], Vc[l, b, h, Lc] = kn[l, b, h], vn[l, b, h]
+            lens_c += 1
+            oracle.decode_batch(qd, Kc, Vc, lens_c, sw.scale())
+        t_dec = time.perf_counter() - t0
+        t_pen = t_ppl = 0.0
+        if wl.vocab:
+            t0 = time.perf_counter()
+            oracle.reflect_penalty(self.z, self.ids, self.rw, wl.tau_l, wl.tau_h, wl.beta)
+            t_pen = time.perf_counter() - t0
+            t0 = time.perf_counter()
+            oracle.answer_ppl(self.za, self.tok, None, wl.tau_p)
+            t_ppl = time.perf_counter() - t0
+        return {"compress_s": t_comp, "decode_s": t_dec, "penalty_s": t_pen, "ppl_s": t_ppl,
+                "total_s": t_comp + t_dec + t_pen + t_ppl}
+
+    def project(self, m):
+        """Measured pieces -> one full step (linear in units, decode steps and rows)."""
+        wl, sw = self.wl, self.sw
+        f = sw.units / wl.units
+        t_comp = m["compress_s"] / f
+        t_dec = (m["decode_s"] / max(self.n_dec, 1)) * wl.decode_steps / f if self.n_dec else 0.0
+        t_voc = m["penalty_s"] * wl.decode_steps + m["ppl_s"] * wl.batch / sw.batch if wl.vocab else 0.0
+        full = t_comp + t_dec + t_voc
+        tokens = wl.batch * (wl.L + wl.decode_steps)
+        return {"full_step_s": full, "value": tokens / full,
+                "compress_tokens_s": wl.batch * wl.L / t_comp,
+                "decode_tokens_s": wl.batch * wl.decode_steps / t_dec if t_dec > 0 else None,
+                "sample_tokens": tokens * m["total_s"] / full}
+
+    def describe(self):
+        wl, sw = self.wl, self.sw
+        return (f"{sw.units} of {wl.units} units ({sw.layers} layer(s) x {sw.batch} sequences x {sw.h_kv} KV heads) "
+                f"at full length: score+select+compact, then {self.n_dec} of {wl.decode_steps} decode steps over them"
+                + ("; penalty once on the full logits; PPL on the sampled sequences" if wl.vocab else "")
+                + "; measured pieces scaled linearly to one full step")
+
+
+def cpu_rate(wl, units, dec_steps, threads=None):
+    """One timed pass of the oracle sample; returns the cpu_baseline-style record."""
     import oracle
-    from paper_2608_04771_gb300 import workloads as W
-    oracle.build()
-    Bs = max(1, min(wl.batch, units_sample // wl.h_kv))
-    sw = wl.reduced(layers=1, batch=Bs)
-    n_units = sw.units
-    K, V = W.make_cache(sw, "cpu", canary=False)
-    Kn, Vn = K.float().numpy(), V.float().numpy()
-    q = W.make_qwin(sw, "cpu").float().numpy()
-    lens = np.full((1, Bs, sw.h_kv), sw.L, np.int32)
-    hist = W.make_reward_history(wl)[:Bs]
-    keep = np.array([oracle.keep_count(oracle.retention_ratio(hist[b], wl.base, wl.delta), wl.L, wl.w)
-                     for b in range(Bs)], np.int32)
-    t0 = time.perf_counter()
-    sc = oracle.score_cache(q, Kn, lens, sw.w, sw.pool, sw.scale())
-    idx = oracle.select_batch(sc.astype(np.float32), lens, keep, sw.w)
-    Kc = np.zeros_like(Kn)
-    Vc = np.zeros_like(Vn)
-    for b in range(Bs):
-        for h in range(sw.h_kv):
-            m = int(keep[b])
-            Kc[0, b, h, :m] = oracle.gather_unit(Kn[0, b, h], idx[0, b, h, :m])
-            Vc[0, b, h, :m] = oracle.gather_unit(Vn[0, b, h], idx[0, b, h, :m])
-    t_comp = time.perf_counter() - t0
-    lens_c = np.broadcast_to(keep.reshape(1, -1, 1), lens.shape).copy()
-    n_dec = min(dec_steps_sample, wl.decode_steps)
-    t0 = time.perf_counter()
-    for s in range(n_dec):
-        qd, kn, vn = W.make_decode_step(sw, s, "cpu")
-        knn, vnn = kn.float().numpy(), vn.float().numpy()
-        for b in range(Bs):
-            for h in range(sw.h_kv):
-                Lc = lens_c[0, b, h]
-                Kc[0, b, h, Lc], Vc[0, b, h, Lc] = knn[0, b, h], vnn[0, b, h]
-        lens_c += 1
-        oracle.decode_batch(qd.float().numpy(), Kc, Vc, lens_c, sw.scale())
-    t_dec = (time.perf_counter() - t0) / max(n_dec, 1)
-    t_voc = 0.0
-    if wl.vocab:
-        z = W.make_vocab_logits(wl, "cpu").numpy()
-        ids = W.make_reflection_ids(wl)
-        t0 = time.perf_counter()
-        oracle.reflect_penalty(z, ids, W.make_reward_history(wl)[:, -1])
-        t_pen = time.perf_counter() - t0
-        za, tok = W.make_answer(wl.reduced(batch=Bs), "cpu")
-        t0 = time.perf_counter()
-        oracle.answer_ppl(za.numpy(), tok.numpy(), None, wl.tau_p)
-        t_ppl = (time.perf_counter() - t0) * wl.batch / Bs
-        t_voc = t_pen * wl.decode_steps + t_ppl
-    scale_units = wl.units / n_units
-    full = t_comp * scale_units + t_dec * scale_units * wl.decode_steps + t_voc
-    desc = (f"{n_units} of {wl.units} units (layer 0, {Bs} sequences) at full length: score+select+compact, "
-            f"{n_dec} of {wl.decode_steps} decode steps; penalty on the full logits; PPL on {Bs} of "
-            f"{wl.batch} sequences; extrapolated linearly to one full step")
-    return full, desc
+    smp = OracleSample(wl, units, dec_steps)
+    if threads:
+        oracle.set_threads(threads)
+    try:
+        m = smp.run()
+        cores = oracle.threads()
+    finally:
+        if threads:
+            oracle.set_threads(int(os.environ["OMP_NUM_THREADS"]))
+    p = smp.project(m)
+    return {"value": p["value"], "unit": UNIT, "cores": cores, "kind": "oracle", "sample": smp.describe(),
+            "extrapolated": smp.sw.units < wl.units or smp.n_dec < wl.decode_steps,
+            "units_timed": smp.sw.units, "units_total": wl.units, "decode_steps_timed": smp.n_dec,
+            "decode_steps_total": wl.decode_steps, "measured_s": m, "projected_full_step_s": p["full_step_s"],
+            "compress_tokens_s": p["compress_tokens_s"], "decode_tokens_s": p["decode_tokens_s"]}
 
 
 def run_reference(args, wl):
-    world, rank, _ = int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")), 0
+    """The reference arm: the oracle as it stands, each step one pass over the bounded sample
+    (timed as it ran); value = the sample's token-equivalents per second of its run."""
+    rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    tokens = wl.batch * (wl.L + wl.decode_steps)
-    times = []
+    import oracle
+    smp = OracleSample(wl, args.ref_units, args.ref_dec_steps)
+    oracle.set_threads(int(os.environ["OMP_NUM_THREADS"]))
+    runs = []
     for i in range(args.warmup + args.steps):
-        t, desc = oracle_sample(wl, args.ref_units, args.ref_dec_steps)
+        m = smp.run()
         if i >= args.warmup:
-            times.append(t)
-    t = statistics.mean(times)
-    value = tokens / t
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
+            runs.append(m)
+    mean = {k: statistics.mean(r[k] for r in runs) for k in runs[0]}
+    p = smp.project(mean)
+    ms = mean["total_s"] * 1e3
+    cores = oracle.threads()
+    desc = smp.describe()
+    line = {"impl": "reference", "metric": METRIC, "value": p["value"], "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": workload_name(wl), "tokens_per_step": tokens},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
-            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "config": {"workload": workload_name(wl), "tokens_per_step": p["sample_tokens"],
+                       "step": "one pass of the oracle over the bounded sample below (not a full step): "
+                               "ms_per_step is that pass as measured, tokens_per_step its token-equivalents "
+                               "(the full step's tokens times its share of the projected full-step time)",
+                       "full_step_tokens": wl.batch * (wl.L + wl.decode_steps),
+                       "projected_full_step_ms": p["full_step_s"] * 1e3},
+            "compress_tokens_s": p["compress_tokens_s"], "decode_tokens_s": p["decode_tokens_s"],
+            "cpu_baseline": {"value": p["value"], "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                             "extrapolated": smp.sw.units < wl.units or smp.n_dec < wl.decode_steps,
+                             "units_timed": smp.sw.units, "units_total": wl.units,
+                             "decode_steps_timed": smp.n_dec, "decode_steps_total": wl.decode_steps,
+                             "measured_s": mean},
+            "e2e": {"value": p["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
@@ -390,7 +471,7 @@ def run_gpu(args, wl):
     reco.reco_check()
     torch.cuda.synchronize()
 
-    ph = {k: [] for k in ("score", "select", "decode", "ppl", "step")}
+    ph = {k: [] for k in ("score", "select", "compact", "decode", "decode_phase", "ppl", "step")}
     # an event pair around every 4th decode launch: the sampled launches give the average
     # launch time (their own algorithmic bytes over their own durations), with a quarter
     # of the event gaps inside the step
@@ -401,12 +482,14 @@ def run_gpu(args, wl):
     with ClockSampler(torch.cuda.current_device()) as clk:
         for _ in range(steps):
             hp.reset()
-            e0, e1, e2, e3, e4 = ev(), ev(), ev(), ev(), ev()
-            e0.record(stream)
-            reco.reco_score_cache(hp.kv, hp.q_win, hp.lens, wl.w, wl.pool, wl.scale(), hp.scores, hp.ws_score)
-            e1.record(stream)
-            reco.reco_select_compact(hp.kv, hp.scores, hp.lens, hp.keep, wl.w, hp.kept, hp.ws_select)
-            e2.record(stream)
+            e = [ev() for _ in range(6)]
+            e[0].record(stream)
+            hp.score()
+            e[1].record(stream)
+            hp.select()
+            e[2].record(stream)
+            hp.compact()
+            e[3].record(stream)
             for s in range(wl.decode_steps):
                 if s in dec_ev:
                     dec_ev[s][0].record(stream)
@@ -415,16 +498,18 @@ def run_gpu(args, wl):
                     dec_ev[s][1].record(stream)
                 if hp.has_vocab:
                     hp.penalty()
-            e3.record(stream)
+            e[4].record(stream)
             if hp.has_vocab:
                 hp.probe()
-            e4.record(stream)
-            e4.synchronize()
-            ph["score"].append(e0.elapsed_time(e1))
-            ph["select"].append(e1.elapsed_time(e2))
+            e[5].record(stream)
+            e[5].synchronize()
+            ph["score"].append(e[0].elapsed_time(e[1]))
+            ph["select"].append(e[1].elapsed_time(e[2]))
+            ph["compact"].append(e[2].elapsed_time(e[3]))
             ph["decode"].append([dec_ev[s][0].elapsed_time(dec_ev[s][1]) for s in sampled])
-            ph["ppl"].append(e3.elapsed_time(e4))
-            ph["step"].append(e0.elapsed_time(e4))
+            ph["decode_phase"].append(e[3].elapsed_time(e[4]))
+            ph["ppl"].append(e[4].elapsed_time(e[5]))
+            ph["step"].append(e[0].elapsed_time(e[5]))
         torch.cuda.synchronize()
         barrier(world)
     reco.reco_check()
@@ -438,14 +523,29 @@ def run_gpu(args, wl):
     dec_bytes = np.array(alg["decode_bytes"])[sampled]
     dec_avg_ms = float(dec_ms.mean())
     dec_achieved = float(dec_bytes.mean() / (dec_avg_ms / 1e3) / 1e9)
-    traffic = decode_traffic(wl.dtype)
+    traffic, traffic_src = decode_traffic(wl)
     score_ms = statistics.mean(ph["score"])
     select_ms = statistics.mean(ph["select"])
+    compact_ms = statistics.mean(ph["compact"])
+    compress_ms = max_over_ranks(score_ms + select_ms + compact_ms, world)
+    decode_ms = max_over_ranks(dec_avg_ms * wl.decode_steps, world)
+    mx = int(hp.keep_host.max())  # rows whose source is another row (kept[r] != r): the ones that move
+    r_ = torch.arange(mx, device=dev, dtype=torch.int32)
+    moved = int(((hp.kept[..., :mx] != r_) & (r_.view(1, 1, 1, -1) < hp.keep.view(1, -1, 1, 1))).sum())
+    compact_gbs = alg["compact_bytes"] / compact_ms / 1e6
     kernels = {
         "score": {"ms": score_ms, "GB/s": alg["score_bytes"] / score_ms / 1e6,
-                  "TFLOP/s": alg["score_flops"] / score_ms / 1e9},
-        "select_compact": {"ms": select_ms, "GB/s": (alg["select_bytes"] + alg["compact_bytes"]) / select_ms / 1e6},
+                  "TFLOP/s": alg["score_flops"] / score_ms / 1e9,
+                  "tensor_frac": alg["score_flops"] / score_ms / 1e9 / tc_burst,
+                  "note": "one logical QK^T pass of flops; the kernel runs two passes over K"},
+        "select": {"ms": select_ms, "GB/s": alg["select_bytes"] / select_ms / 1e6},
+        "compact": {"ms": compact_ms, "GB/s": compact_gbs, "frac": compact_gbs / hbm, "peak": hbm,
+                    "peak_kind": peak_kind, "frac_of_8TBs": compact_gbs / 8000.0,
+                    "algorithmic_bytes": alg["compact_bytes"],
+                    "rows_moved_frac": moved / max(1, int(hp.keep_host.sum()) * wl.layers * wl.h_kv),
+                    "timing": "own event pair in the step (reco_compact after reco_select_topm)"},
         "decode": {"ms_per_launch": dec_avg_ms, "GB/s": dec_achieved, "launches": wl.decode_steps,
+                   "phase_ms": statistics.mean(ph["decode_phase"]),
                    "timed_launches": f"every 4th ({len(sampled)} of {wl.decode_steps}) between CUDA events"},
     }
     if hp.has_vocab:
@@ -460,24 +560,31 @@ def run_gpu(args, wl):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        t_full, desc = oracle_sample(wl, args.ref_units, args.ref_dec_steps)
-        cpu = {"value": tokens / t_full, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]),
-               "kind": "oracle", "sample": desc}
+        from paper_2608_04771_gb300 import workloads as W
+        cpu = cpu_rate(wl, args.ref_units, args.ref_dec_steps)
+        # one host core, on the Tiny workload (whole) and on a sample of the 1.5B-class stack
+        cpu["one_core"] = {name: cpu_rate(W.WORKLOADS[name], u, n, threads=1)
+                           for name, u, n in (("tiny", 2, 1), ("1.5b", 8, 8))}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps, "warmup": warm,
             "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+            "compress_tokens_s": world * wl.batch * wl.L / (compress_ms / 1e3),
+            "decode_tokens_s": world * wl.batch * wl.decode_steps / (decode_ms / 1e3),
             "config": {"workload": workload_name(wl), "tokens_per_step": tokens,
                        "parallelism": f"replicas x{world} (sequences sharded, no collective)",
-                       "l2": "inputs larger than L2 (K/V 7.5 GB at 7B); the cache restore before each step "
-                             "(outside the timed events) also overwrites L2",
+                       "l2": f"inputs larger than L2 (K/V {2 * hp.K.numel() * hp.K.element_size() / 1e9:.1f} GB); "
+                             "the cache restore before each step (outside the timed events) also overwrites L2",
+                       "rates": "compress_tokens_s = B*L / (score + select + compact); decode_tokens_s = "
+                                "B*steps / (steps * mean decode launch), attention only",
                        "kernels": kernels, "keep_counts": [int(x) for x in hp.keep_host]},
-            "roofline": {"bound": "hbm", "kernel": "decode_mma (reco_decode_attn)", "achieved": dec_achieved,
+            "roofline": {"bound": "hbm", "kernel": "decode_tma (reco_decode_attn)", "achieved": dec_achieved,
                          "peak": hbm, "unit": "GB/s", "frac": dec_achieved / hbm, "peak_kind": peak_kind,
                          "frac_of_8TBs": dec_achieved / 8000.0,
-                         "traffic": traffic, "algorithmic_bytes_per_launch": float(dec_bytes.mean())},
+                         "traffic": traffic, "traffic_source": traffic_src,
+                         "algorithmic_bytes_per_launch": float(dec_bytes.mean())},
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": hp.launches_per_step() * steps,
@@ -489,22 +596,54 @@ def run_gpu(args, wl):
         dist.destroy_process_group()
 
 
+def gpu_local_cpus(dev):
+    """Host CPUs attached to the GPU's NUMA node (from sysfs), or None if not visible."""
+    try:
+        pr = torch.cuda.get_device_properties(dev)
+        bus = f"{pr.pci_domain_id:04x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+        text = open(f"/sys/bus/pci/devices/{bus}/local_cpulist").read().strip()
+    except Exception:
+        return None
+    cpus = set()
+    for part in text.split(","):
+        if "-" in part:
+            lo, hi = part.split("-")
+            cpus.update(range(int(lo), int(hi) + 1))
+        elif part:
+            cpus.add(int(part))
+    allowed = os.sched_getaffinity(0)
+    return (cpus & allowed) or None
+
+
 def run_e2e(hp, wl, args, world):
     """Same metric through the C ABI with host buffers: every step copies all of its inputs
     from pinned host memory, runs the hot path and reads its results back, all inside the
     timed region.  The steps are pipelined over two device buffer sets: step i+1's inputs
     travel on a copy stream while step i computes, and a set is overwritten only after the
-    step that last used it has finished (its results read back)."""
+    step that last used it has finished (its results read back).  The pinned buffers are
+    allocated and first touched from the CPUs local to the GPU when sysfs names them, so
+    their pages sit on the GPU's own host memory node."""
     from paper_2608_04771_gb300 import driver
     dev = hp.K.device
-    pin = lambda t: t.detach().cpu().pin_memory()  # noqa: E731
-    host = dict(K=pin(hp.K0), V=pin(hp.V0), lens=pin(hp.lens0), q_win=pin(hp.q_win), keep=pin(hp.keep),
-                dq=pin(hp.dq), dk=pin(hp.dk), dv=pin(hp.dv))
-    if hp.has_vocab:
-        host.update(logits=pin(hp.logits), ids=pin(hp.ids), rewards=pin(hp.rewards),
-                    ans_logits=pin(hp.ans_logits), ans_tokens=pin(hp.ans_tokens))
-    out_names = ["out"] + (["ppl", "stop"] if hp.has_vocab else [])
-    host_out = {k: torch.empty_like(getattr(hp, k), device="cpu").pin_memory() for k in out_names}
+    local = gpu_local_cpus(dev)
+    prev_aff = os.sched_getaffinity(0)
+    if local:
+        os.sched_setaffinity(0, local)
+    try:
+        def pin(t):  # device tensor -> a pinned host copy, with no pageable intermediate
+            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            h.copy_(t)
+            return h
+        host = dict(K=pin(hp.K0), V=pin(hp.V0), lens=pin(hp.lens0), q_win=pin(hp.q_win), keep=pin(hp.keep),
+                    dq=pin(hp.dq), dk=pin(hp.dk), dv=pin(hp.dv))
+        if hp.has_vocab:
+            host.update(logits=pin(hp.logits), ids=pin(hp.ids), rewards=pin(hp.rewards),
+                        ans_logits=pin(hp.ans_logits), ans_tokens=pin(hp.ans_tokens))
+        out_names = ["out"] + (["ppl", "stop"] if hp.has_vocab else [])
+        host_out = {k: torch.empty(getattr(hp, k).shape, dtype=getattr(hp, k).dtype, pin_memory=True)
+                    for k in out_names}
+    finally:
+        os.sched_setaffinity(0, prev_aff)
     sets = [hp, driver.HotPath(wl, dev, out_dtype=hp.out.dtype, keep_pristine=False)]
     h2d = sum(h.numel() * h.element_size() for h in host.values())
     d2h = sum(h.numel() * h.element_size() for h in host_out.values())
@@ -514,15 +653,23 @@ def run_e2e(hp, wl, args, world):
     ready = [torch.cuda.Event() for _ in sets]
     done = [torch.cuda.Event() for _ in sets]
     free = [torch.cuda.Event() for _ in sets]
+    cp_ev = []
 
-    def enqueue(i):
+    def enqueue(i, timed=False):
         s = sets[i % 2]
         with torch.cuda.stream(cps):
             if i >= 2:
                 cps.wait_event(free[i % 2])  # the step that last used this set has finished
+            if timed:
+                c0 = torch.cuda.Event(enable_timing=True)
+                c0.record(cps)
             for k, h in host.items():
                 getattr(s, k).copy_(h, non_blocking=True)
             ready[i % 2].record(cps)
+            if timed:
+                c1 = torch.cuda.Event(enable_timing=True)
+                c1.record(cps)
+                cp_ev.append((c0, c1))
         comp.wait_event(ready[i % 2])
         s.step()
         done[i % 2].record(comp)
@@ -540,14 +687,17 @@ def run_e2e(hp, wl, args, world):
     a.record(comp)
     cps.wait_event(a)
     for i in range(n):
-        enqueue(i)
+        enqueue(i, timed=True)
     comp.wait_stream(dps)  # the last results read back
     b.record(comp)
     b.synchronize()
     ms = max_over_ranks(a.elapsed_time(b) / n, world)
+    cp_ms = statistics.median(c0.elapsed_time(c1) for c0, c1 in cp_ev)
     tokens = wl.batch * (wl.L + wl.decode_steps)
     return {"value": world * tokens / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n,
+            "h2d_GBps": h2d / cp_ms / 1e6, "h2d_ms_per_step": cp_ms,
+            "pinned_near_gpu": bool(local),
             "schedule": "two device buffer sets and three streams: step i+1's host-to-device copies and step "
                         "i-1's read-back overlap step i's compute"}
 
@@ -609,13 +759,13 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
-    ap.add_argument("--workload", default="7b", choices=["tiny", "1.5b", "7b", "32b", "trace"])
+    ap.add_argument("--workload", default="32b", choices=["tiny", "1.5b", "7b", "32b", "trace"])
     ap.add_argument("--reading", default="A", choices=["A", "B"], help="trace: budget base reading")
     ap.add_argument("--generated", type=int, default=0, help="trace: generated tokens (default 8192)")
     ap.add_argument("--no-graph", action="store_true", help="trace: per-token calls without a CUDA graph")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--ref-units", type=int, default=32, help="oracle sample: units of layer 0")
+    ap.add_argument("--ref-units", type=int, default=16, help="oracle sample: units (whole layers, or part of layer 0)")
     ap.add_argument("--ref-dec-steps", type=int, default=8, help="oracle sample: decode steps")
     ap.add_argument("--layers", type=int, help="override the layer count (profiling a smaller case)")
     ap.add_argument("--batch", type=int, help="override the batch (profiling a smaller case)")

@@ -184,6 +184,37 @@ reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t 
                                 const int32_t *keep, int w, int32_t *kept_idx, void *ws,
                                 size_t ws_bytes, cudaStream_t stream);
 
+/* The two halves of reco_select_compact as separate calls, for callers that want the
+ * kept indices before the cache moves (for example to compact per-token state of their
+ * own with the same indices) or that time the two steps apart.
+ * reco_select_topm writes exactly the `kept` that reco_select_compact computes (Sec. 3.2:
+ * the m-w best candidates, ties to the lower index, then the window, ascending) into the
+ * first keep[b] entries of each unit of kept_idx, and changes nothing else: K, V and lens
+ * are left as they are.
+ *   scores, lens, keep, w : as reco_select_compact (lens is only read)
+ *   kept_idx : [n_layers][B][H_kv][L_cap] int32 (device, written; required)
+ *   ws       : workspace of reco_workspace_bytes(RECO_OP_SELECT, kv, w) bytes
+ * A unit with an out-of-range length or keep count gets no indices (device error word
+ * set).  The kv pointers may be NULL: the cache is not touched.                     */
+reco_status reco_select_topm(const reco_kv *kv, const float *scores, const int32_t *lens, const int32_t *keep,
+                             int w, int32_t *kept_idx, void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* In-place compaction of every unit to the rows kept_idx names (Sec. 3.2, the cache
+ * compressed from L to m_i tokens): with L = lens[unit] and m = keep[b],
+ *   K[unit, r] = K[unit, kept_idx[unit, r]] and V likewise for r < m, lens[unit] = m,
+ * for each unit with w <= m < L; m == L leaves the unit as it is.  No workspace.
+ *   kept_idx : [n_layers][B][H_kv][L_cap] int32 (device), e.g. from reco_select_topm.
+ *              Entry r must lie in [r, L): any strictly increasing list of rows below L
+ *              qualifies.  Row r's source is then never a row an earlier destination
+ *              overwrote, so the copy in place is exact.  An entry outside [r, L) is not
+ *              copied and sets the device error word.
+ *   lens     : [n_layers][B][H_kv] int32 (device, in: L, out: m)
+ *   keep     : [B] int32 (device)
+ * A unit with lens outside [w, L_cap] or keep outside [w, lens] is left untouched (device
+ * error word set).                                                                   */
+reco_status reco_compact(const reco_kv *kv, const int32_t *kept_idx, int32_t *lens, const int32_t *keep, int w,
+                         cudaStream_t stream);
+
 /* Decode attention over the ragged compacted cache: the per-token attention whose
  * cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2, main results).
  * If k_new and v_new are both non-NULL, each unit first appends its new row at

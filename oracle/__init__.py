@@ -63,6 +63,10 @@ def _load():
 def _bind(lib):
     """Declare the C signatures on a loaded oracle library."""
     c_int, c_double, c_float = ctypes.c_int, ctypes.c_double, ctypes.c_float
+    lib.oracle_set_threads.argtypes = [c_int]
+    lib.oracle_set_threads.restype = None
+    lib.oracle_threads.argtypes = []
+    lib.oracle_threads.restype = c_int
     lib.oracle_retention_ratio.argtypes = [_f32p, c_int, c_double, c_double]
     lib.oracle_retention_ratio.restype = c_double
     lib.oracle_keep_count.argtypes = [c_double, c_int, c_int]
@@ -110,6 +114,15 @@ def _i32(a):
 
 
 # ---- Eq. 1 -----------------------------------------------------------------
+def set_threads(n: int) -> None:
+    """Threads of the OpenMP loops over units (timing plumbing; results do not depend on it)."""
+    _load().oracle_set_threads(int(n))
+
+
+def threads() -> int:
+    return int(_load().oracle_threads())
+
+
 def retention_ratio(rewards, base: float = 0.25, delta: float = 0.1) -> float:
     r = _f32(rewards).ravel()
     return float(_load().oracle_retention_ratio(r, int(r.size), float(base), float(delta)))

@@ -38,6 +38,29 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Timing plumbing, no arithmetic: the number of threads the OpenMP loops of the
+ * batched wrappers use (the benchmark times the oracle on one core and on all). */
+void oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    omp_set_num_threads(n > 0 ? n : 1);
+#else
+    (void)n;
+#endif
+}
+
+int oracle_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
 
 /* ------------------------------------------------------------------------- */
 /* Eq. 1 (Sec. 3.2, "Reward-driven retention"): lambda_i = lambda - delta *   */

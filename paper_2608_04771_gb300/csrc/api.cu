@@ -309,6 +309,38 @@ reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t 
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_select_compact launch");
 }
 
+reco_status reco_select_topm(const reco_kv *kv, const float *scores, const int32_t *lens, const int32_t *keep, int w,
+                             int32_t *kept_idx, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    reco_status st = check_kv(kv, false);
+    if (st != RECO_OK) return st;
+    if (!scores || !lens || !keep || !kept_idx) return fail(RECO_EINVAL, "NULL scores, lens, keep or kept_idx");
+    if (((uintptr_t)scores & 3u) || ((uintptr_t)lens & 3u) || ((uintptr_t)keep & 3u) || ((uintptr_t)kept_idx & 3u))
+        return fail(RECO_EINVAL, "scores, lens, keep and kept_idx must be 4-byte aligned");
+    if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
+    reco::SelectWs lay = reco::select_ws_layout(*kv, ws);
+    if ((st = check_ws(ws, ws_bytes, lay.bytes)) != RECO_OK) return st;
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_select_only(*kv, scores, lens, keep, w, kept_idx, lay, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_select_topm launch");
+}
+
+reco_status reco_compact(const reco_kv *kv, const int32_t *kept_idx, int32_t *lens, const int32_t *keep, int w,
+                         cudaStream_t stream)
+{
+    reco_status st = check_kv(kv);
+    if (st != RECO_OK) return st;
+    if (!kept_idx || !lens || !keep) return fail(RECO_EINVAL, "NULL kept_idx, lens or keep");
+    if (((uintptr_t)lens & 3u) || ((uintptr_t)keep & 3u) || ((uintptr_t)kept_idx & 3u))
+        return fail(RECO_EINVAL, "lens, keep and kept_idx must be 4-byte aligned");
+    if (w < 1 || w > kv->L_cap) return fail(RECO_EINVAL, "window w=%d outside [1, L_cap=%d]", w, kv->L_cap);
+    unsigned *err;
+    if ((st = error_word(&err)) != RECO_OK) return st;
+    cudaError_t e = reco::launch_compact(*kv, kept_idx, lens, keep, w, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_compact launch");
+}
+
 reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new, const void *v_new, int32_t *lens,
                              float scale, void *out, reco_dtype out_dtype, float *lse, void *ws, size_t ws_bytes,
                              cudaStream_t stream)
@@ -425,6 +457,7 @@ extern "C" reco_status reco_answer_ppl_static(const float *logits, const int32_t
                                               cudaStream_t stream)
 {
     if (B < 1 || n < 0 || V < 1) return fail(RECO_EINVAL, "need B >= 1, n >= 0, V >= 1");
+    if (B > 65535 || n > 65535) return fail(RECO_EUNSUPPORTED, "B or n exceeds 65535");
     if ((long long)B * n > RECO_PPL_STATIC_MAX_ROWS)
         return fail(RECO_EINVAL, "B*n = %lld answer rows exceed the static scratch of %d rows", (long long)B * n,
                     RECO_PPL_STATIC_MAX_ROWS);

@@ -74,6 +74,10 @@ cudaError_t launch_lse_push(const float *lse, long n, float *ring, int slots, lo
 cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
                                   const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
                                   unsigned *err, cudaStream_t s);
+cudaError_t launch_select_only(const reco_kv &kv, const float *scores, const int32_t *lens, const int32_t *keep,
+                               int w, int32_t *kept_idx, const SelectWs &ws, unsigned *err, cudaStream_t s);
+cudaError_t launch_compact(const reco_kv &kv, const int32_t *kept_idx, int32_t *lens, const int32_t *keep, int w,
+                           unsigned *err, cudaStream_t s);
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
                           int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
                           const DecodeWs &ws, unsigned *err, cudaStream_t s);

@@ -12,8 +12,8 @@
 // still matches the prefix (in the later passes, few do).
 //
 // compact_rows: one CTA per (unit, K|V, 128-byte column slice).  kept[] is strictly
-// increasing, so kept[r] >= r: the source of destination r is never a row that an
-// earlier destination overwrote.  Each CTA walks its destinations in order, reads a
+// increasing, so kept[r] >= r (the kernel refuses any index that is not): the source
+// of destination r is never a row that an earlier destination overwrote.  Each CTA walks its destinations in order, reads a
 // chunk of source rows, synchronises, then writes the chunk; reads of later chunks
 // may run ahead of earlier writes because their sources lie above every row written
 // so far.  Rows with kept[r] == r are not moved.
@@ -76,8 +76,8 @@ __device__ __forceinline__ int block_scan_flag(bool flag, int *tot, int &total)
 }
 
 template <int NT>
-__global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scores, int32_t *lens,
-                                                  const int32_t *__restrict__ keep, int w, int B, int Hkv,
+__global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scores, const int32_t *lens,
+                                                  int32_t *lens_out, const int32_t *__restrict__ keep, int w, int B, int Hkv,
                                                   int L_cap, int32_t *__restrict__ idx_out,
                                                   int32_t *__restrict__ count, unsigned *err)
 {
@@ -180,7 +180,7 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
     for (int t = tid; t < w; t += NT) idx[kc + t] = nc + t;
     if (tid == 0) {
         count[u] = m;
-        lens[u] = m;
+        if (lens_out) lens_out[u] = m;
     }
 }
 
@@ -188,8 +188,8 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
 // flight), the radix passes run from there, and the ordered emit done by warp-contiguous
 // segments: one counting sweep, one scan of the 32 warps' counts, one writing sweep.
 template <int NT>
-__global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__ scores, int32_t *lens,
-                                                       const int32_t *__restrict__ keep, int w, int B, int Hkv,
+__global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__ scores, const int32_t *lens,
+                                                       int32_t *lens_out, const int32_t *__restrict__ keep, int w, int B, int Hkv,
                                                        int L_cap, int32_t *__restrict__ idx_out,
                                                        int32_t *__restrict__ count, unsigned *err)
 {
@@ -333,18 +333,48 @@ __global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__
     for (int t = tid; t < w; t += NT) idx[kc + t] = nc + t;
     if (tid == 0) {
         count[u] = m;
-        lens[u] = m;
+        if (lens_out) lens_out[u] = m;
     }
 }
 
+// Rows to move for unit u.  From the selection: its count (0 = leave the unit alone).
+// From the caller's keep counts: m = keep[b] when w <= m < L <= L_cap; m == L is the
+// no-op; anything else leaves the unit alone and sets the error word.
+// `lim` receives the end of the rows a source index may name.
+struct CountFromSelect {
+    const int32_t *count;
+    int L_cap;
+    __device__ __forceinline__ int rows(long u, unsigned *, int &lim) const
+    {
+        lim = L_cap;
+        return count[u];
+    }
+};
+struct CountFromKeep {
+    const int32_t *lens, *keep;
+    int w, B, Hkv, L_cap;
+    __device__ __forceinline__ int rows(long u, unsigned *err, int &lim) const
+    {
+        const int L = lens[u], m = keep[(u / Hkv) % B];
+        lim = L;
+        if (L < w || L > L_cap || m < w || m > L) {
+            if (blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0)
+                raise_error(err, (L < w || L > L_cap) ? ERR_LEN : ERR_KEEP);
+            return 0;
+        }
+        return m == L ? 0 : m;
+    }
+};
+
+template <class Count>
 __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int32_t *__restrict__ idx_all,
-                                                    const int32_t *__restrict__ count, int L_cap,
-                                                    int row_bytes, unsigned *err)
+                                                    Count cnt, int L_cap, int row_bytes, unsigned *err)
 {
     constexpr int P = 8;  // 16-byte pieces per 128-byte slice
     constexpr int U = 2;  // rows per thread in flight
     const long u = blockIdx.x;
-    const int m = count[u];
+    int lim;
+    const int m = cnt.rows(u, err, lim);
     if (m == 0) return;
     char *base = (blockIdx.y == 0 ? K : V) + u * (long)L_cap * row_bytes;
     const int32_t *idx = idx_all + u * L_cap;
@@ -360,7 +390,7 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
             dst[i] = -1;
             if (r < m) {
                 const int src = idx[r];
-                if (src < r || src >= L_cap) {  // never trust an index outside [r, L_cap)
+                if (src < r || src >= lim) {  // never trust an index outside [r, lim)
                     raise_error(err, ERR_INTERNAL);
                 } else if (src != r) {
                     v[i] = *reinterpret_cast<const uint4 *>(base + (long)src * row_bytes + off);
@@ -375,30 +405,74 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
     }
 }
 
+// lens[u] = keep[b] for the units reco_compact moved (after every CTA of the unit read lens).
+__global__ void compact_set_lens(int32_t *lens, const int32_t *__restrict__ keep, long units, int w, int B,
+                                 int Hkv, int L_cap)
+{
+    const long u = (long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (u >= units) return;
+    const int L = lens[u], m = keep[(u / Hkv) % B];
+    if (L >= w && L <= L_cap && m >= w && m < L) lens[u] = m;
+}
+
+static cudaError_t launch_select(const reco_kv &kv, const float *scores, const int32_t *lens, int32_t *lens_out,
+                                 const int32_t *keep, int w, int32_t *idx, int32_t *count, unsigned *err,
+                                 cudaStream_t s)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    // keys of a unit staged in shared memory when L_cap - w of them fit
+    const size_t key_bytes = (size_t)(kv.L_cap - w) * sizeof(uint32_t);
+    if (key_bytes <= kSelectSmemKeys * sizeof(uint32_t)) {
+        cudaError_t e = cudaFuncSetAttribute(select_topm_smem<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kSelectSmemKeys * (int)sizeof(uint32_t));
+        if (e != cudaSuccess) return e;
+        select_topm_smem<1024><<<(unsigned)units, 1024, key_bytes, s>>>(scores, lens, lens_out, keep, w, kv.B,
+                                                                       kv.H_kv, kv.L_cap, idx, count, err);
+    } else {
+        select_topm<1024><<<(unsigned)units, 1024, 0, s>>>(scores, lens, lens_out, keep, w, kv.B, kv.H_kv,
+                                                           kv.L_cap, idx, count, err);
+    }
+    return cudaGetLastError();
+}
+
+static dim3 compact_grid(const reco_kv &kv, int &row_bytes)
+{
+    row_bytes = kv.d * (kv.dtype == RECO_F32 ? 4 : 2);
+    return dim3((unsigned)((long)kv.n_layers * kv.B * kv.H_kv), 2, row_bytes / 128);
+}
+
 cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,
                                   const int32_t *keep, int w, int32_t *kept_idx, const SelectWs &ws,
                                   unsigned *err, cudaStream_t s)
 {
-    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     int32_t *idx = kept_idx ? kept_idx : ws.idx;
-    // keys of a unit staged in shared memory when L_cap - w of them fit
-    const size_t key_bytes = (size_t)(kv.L_cap - w) * sizeof(uint32_t);
-    cudaError_t e;
-    if (key_bytes <= kSelectSmemKeys * sizeof(uint32_t)) {
-        e = cudaFuncSetAttribute(select_topm_smem<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kSelectSmemKeys * (int)sizeof(uint32_t));
-        if (e != cudaSuccess) return e;
-        select_topm_smem<1024><<<(unsigned)units, 1024, key_bytes, s>>>(scores, lens, keep, w, kv.B, kv.H_kv,
-                                                                       kv.L_cap, idx, ws.count, err);
-    } else {
-        select_topm<1024><<<(unsigned)units, 1024, 0, s>>>(scores, lens, keep, w, kv.B, kv.H_kv, kv.L_cap, idx,
-                                                           ws.count, err);
-    }
-    e = cudaGetLastError();
+    cudaError_t e = launch_select(kv, scores, lens, lens, keep, w, idx, ws.count, err, s);
     if (e != cudaSuccess) return e;
-    const int row_bytes = kv.d * (kv.dtype == RECO_F32 ? 4 : 2);
-    dim3 grid((unsigned)units, 2, row_bytes / 128);
-    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, idx, ws.count, kv.L_cap, row_bytes, err);
+    int row_bytes;
+    const dim3 grid = compact_grid(kv, row_bytes);
+    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, idx, CountFromSelect{ws.count, kv.L_cap}, kv.L_cap,
+                                      row_bytes, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_select_only(const reco_kv &kv, const float *scores, const int32_t *lens, const int32_t *keep,
+                               int w, int32_t *kept_idx, const SelectWs &ws, unsigned *err, cudaStream_t s)
+{
+    return launch_select(kv, scores, lens, nullptr, keep, w, kept_idx, ws.count, err, s);
+}
+
+cudaError_t launch_compact(const reco_kv &kv, const int32_t *kept_idx, int32_t *lens, const int32_t *keep, int w,
+                           unsigned *err, cudaStream_t s)
+{
+    int row_bytes;
+    const dim3 grid = compact_grid(kv, row_bytes);
+    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, kept_idx,
+                                      CountFromKeep{lens, keep, w, kv.B, kv.H_kv, kv.L_cap}, kv.L_cap, row_bytes,
+                                      err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const long units = grid.x;
+    compact_set_lens<<<(unsigned)((units + 255) / 256), 256, 0, s>>>(lens, keep, units, w, kv.B, kv.H_kv, kv.L_cap);
     return cudaGetLastError();
 }
 

@@ -317,7 +317,9 @@ __global__ void __launch_bounds__(NT) ppl_rows(const float *__restrict__ logits,
     if (t >= nb) return;
     const float *z = logits + ((size_t)b * n + t) * V;
     float m = -INFINITY, s = 0.f;
-    if ((V & 3) == 0) {
+    // Vector loads only when every row starts on a 16-byte boundary: the base is
+    // 16-byte aligned and rows are a multiple of 4 floats long.
+    if ((V & 3) == 0 && ((uintptr_t)logits & 15u) == 0) {
         const float4 *z4 = reinterpret_cast<const float4 *>(z);
         for (int i = threadIdx.x; i < V / 4; i += NT) {
             const float4 x = __ldcs(z4 + i);

@@ -3,7 +3,8 @@
 A step is what happens at one reasoning-step boundary and the decode that follows:
   1. Eq. 1 per sequence on the host (library helper) -> keep counts m_b
   2. reco_score_cache      (Eq. 2 scores, all layers in one call)
-  3. reco_select_compact   (top-m per KV head, in-place compaction)
+  3. reco_select_topm, reco_compact  (top-m per KV head, then in-place compaction:
+     reco_select_compact's two halves as separate calls, so they can be timed apart)
   4. for each decode step: reco_decode_attn (append + attention over the ragged
      cache, all layers) and reco_reflect_penalty (Eq. 3-4 on the step's logits)
   5. reco_answer_ppl        (Eq. 5-6 probe over the answer logits)
@@ -71,12 +72,22 @@ class HotPath:
         self.V.copy_(self.V0)
         self.lens.copy_(self.lens0)
 
-    def compress(self, stream=None):
+    def score(self, stream=None):
         wl = self.wl
         reco.reco_score_cache(self.kv, self.q_win, self.lens, wl.w, wl.pool, wl.scale(), self.scores,
                               self.ws_score, stream=stream)
-        reco.reco_select_compact(self.kv, self.scores, self.lens, self.keep, wl.w, self.kept,
-                                 self.ws_select, stream)
+
+    def select(self, stream=None):
+        reco.reco_select_topm(self.kv, self.scores, self.lens, self.keep, self.wl.w, self.kept, self.ws_select,
+                              stream)
+
+    def compact(self, stream=None):
+        reco.reco_compact(self.kv, self.kept, self.lens, self.keep, self.wl.w, stream)
+
+    def compress(self, stream=None):
+        self.score(stream)
+        self.select(stream)
+        self.compact(stream)
 
     def decode(self, s: int, stream=None):
         reco.reco_decode_attn(self.kv, self.dq[s], self.dk[s], self.dv[s], self.lens, self.wl.scale(),
@@ -107,8 +118,8 @@ class HotPath:
             self.probe(stream)
 
     def launches_per_step(self) -> int:
-        """Library kernels launched by one step (the decode's counter reset is a memset)."""
-        n = 4 + 2  # score: pass 1, combine, pass 2, pool; select, compact
+        """Library kernels launched by one step."""
+        n = 4 + 3  # score: pass 1, combine, pass 2, pool; select; compact and its length update
         n += self.wl.decode_steps * (1 + (1 if self.has_vocab else 0))
         n += 2 if self.has_vocab else 0
         return n

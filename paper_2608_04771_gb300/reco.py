@@ -20,8 +20,9 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = ran
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_score_cache_lse", "reco_lse_push", "reco_select_compact", "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample",
-           "reco_answer_ppl", "reco_answer_ppl_static")
+           "reco_score_cache_lse", "reco_lse_push", "reco_select_compact", "reco_select_topm", "reco_compact",
+           "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
+           "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
 
 
@@ -66,6 +67,8 @@ def lib():
     L.reco_score_cache_lse.argtypes = [kvp, vp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_lse_push.argtypes = [vp, ctypes.c_int64, vp, i32, vp, vp]
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
+    L.reco_select_topm.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
+    L.reco_compact.argtypes = [kvp, vp, vp, vp, i32, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
     L.reco_penalty_sample.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp]
@@ -73,6 +76,7 @@ def lib():
     L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
                  "reco_score_cache", "reco_score_cache_lse", "reco_lse_push", "reco_select_compact",
+                 "reco_select_topm", "reco_compact",
                  "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
                  "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
@@ -190,6 +194,17 @@ def reco_select_compact(kv: reco_kv, scores, lens, keep, w: int, kept_idx, ws, s
                                   _ptr(kept_idx), _ptr(ws), ws.numel(), _stream(stream)))
 
 
+def reco_select_topm(kv: reco_kv, scores, lens, keep, w: int, kept_idx, ws, stream=None):
+    """The selection of reco_select_compact alone: kept indices written, cache and lens untouched."""
+    _ok(lib().reco_select_topm(ctypes.byref(kv), _ptr(scores), _ptr(lens), _ptr(keep), int(w), _ptr(kept_idx),
+                               _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def reco_compact(kv: reco_kv, kept_idx, lens, keep, w: int, stream=None):
+    """The compaction of reco_select_compact alone, to the rows kept_idx names."""
+    _ok(lib().reco_compact(ctypes.byref(kv), _ptr(kept_idx), _ptr(lens), _ptr(keep), int(w), _stream(stream)))
+
+
 def reco_decode_attn(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, lse, ws, stream=None):
     _ok(lib().reco_decode_attn(ctypes.byref(kv), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(lens),
                                float(scale), _ptr(out), _dtype_code(out.dtype), _ptr(lse), _ptr(ws),
@@ -218,14 +233,26 @@ def reco_penalty_sample(logits, ids, rewards, uniforms, tokens, ws, tau_l=0.4, t
                                   ws.numel(), _stream(stream)))
 
 
-def reco_answer_ppl(logits, tokens, n_valid, tau_p, ppl, stop, ws, stream=None):
+def _ppl_args(logits, tokens, n_valid):
+    """[B, n, V] float32 logits and [B, n] int32 tokens, both contiguous (strides are not passed)."""
+    if logits.dim() != 3 or logits.dtype != torch.float32 or not logits.is_contiguous():
+        raise ValueError("logits must be a contiguous float32 [B, n, V] tensor")
     B, n, V = logits.shape
+    if tokens.shape != (B, n) or tokens.dtype != torch.int32 or not tokens.is_contiguous():
+        raise ValueError("tokens must be a contiguous int32 [B, n] tensor")
+    if n_valid is not None and (n_valid.numel() != B or n_valid.dtype != torch.int32 or not n_valid.is_contiguous()):
+        raise ValueError("n_valid must be a contiguous int32 [B] tensor")
+    return B, n, V
+
+
+def reco_answer_ppl(logits, tokens, n_valid, tau_p, ppl, stop, ws, stream=None):
+    B, n, V = _ppl_args(logits, tokens, n_valid)
     _ok(lib().reco_answer_ppl(_ptr(logits), _ptr(tokens), _ptr(n_valid), B, n, V, float(tau_p),
                               _ptr(ppl), _ptr(stop), _ptr(ws), ws.numel(), _stream(stream)))
 
 
 def reco_answer_ppl_static(logits, tokens, n_valid, tau_p, ppl, stop, stream=None):
     """reco_answer_ppl without a workspace: the library's fixed scratch array is used."""
-    B, n, V = logits.shape
+    B, n, V = _ppl_args(logits, tokens, n_valid)
     _ok(lib().reco_answer_ppl_static(_ptr(logits), _ptr(tokens), _ptr(n_valid), B, n, V, float(tau_p),
                                      _ptr(ppl), _ptr(stop), _stream(stream)))

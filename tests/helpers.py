@@ -63,6 +63,18 @@ def gpu_select(wl, K, V, scores, lens, keep):
     return kept
 
 
+def gpu_select_split(wl, K, V, scores, lens, keep):
+    """reco_select_topm, then reco_compact on the indices it wrote (the two halves of
+    reco_select_compact as separate calls)."""
+    kv = reco.make_kv(K, V, wl.h_q)
+    kept = torch.full(K.shape[:4], -1, dtype=torch.int32, device=K.device)
+    ws = reco.workspace(reco.RECO_OP_SELECT, kv, wl.w, K.device)
+    keep_t = torch.as_tensor(keep, dtype=torch.int32, device=K.device)
+    reco.reco_select_topm(kv, scores, lens, keep_t, wl.w, kept, ws)
+    reco.reco_compact(kv, kept, lens, keep_t, wl.w)
+    return kept
+
+
 def gpu_decode(wl, K, V, lens, q, k_new=None, v_new=None, out_dtype=torch.float32):
     kv = reco.make_kv(K, V, wl.h_q)
     out = torch.empty(q.shape, dtype=out_dtype, device=q.device)

@@ -20,11 +20,15 @@ def _lib():
     reco.lib()
 
 
-@pytest.mark.parametrize("name", ["7b", "1.5b", "32b"])
-def test_full_size_sampled_units(name):
+@pytest.mark.parametrize("name,out_dtype", [("32b", torch.bfloat16), ("7b", torch.bfloat16), ("1.5b", torch.bfloat16),
+                                            ("7b", torch.float32)])
+def test_full_size_sampled_units(name, out_dtype):
+    """bf16 output is what bench.py runs (driver.HotPath's default); fp32 output checks the
+    same launch at the tighter bar."""
     wl = W.WORKLOADS[name]
-    hp = driver.HotPath(wl, DEV, out_dtype=torch.float32, keep_pristine=False)
-    units = [(0, 0, 0), (wl.layers // 2, wl.batch // 2, wl.h_kv - 1), (wl.layers - 1, wl.batch - 1, wl.h_kv // 2)]
+    hp = driver.HotPath(wl, DEV, out_dtype=out_dtype, keep_pristine=False)
+    units = [(0, 0, 0), (wl.layers // 2, wl.batch // 2, wl.h_kv - 1), (wl.layers - 1, wl.batch - 1, wl.h_kv // 2),
+             (1, wl.batch - 1, 0), (wl.layers - 2, 0, wl.h_kv - 1)]
     G = wl.G
     saved = {}
     for (l, b, h) in units:
@@ -34,7 +38,8 @@ def test_full_size_sampled_units(name):
     hp.step()
     reco.reco_check()
     torch.cuda.synchronize()
-    check_steps = sorted({0, wl.decode_steps // 2, wl.decode_steps - 1})
+    check_steps = sorted({0, 1, wl.decode_steps // 2, wl.decode_steps - 1})
+    atol = DECODE_ATOL[wl.dtype]
     for (l, b, h) in units:
         K0, V0, q = saved[(l, b, h)]
         m = int(hp.keep_host[b])
@@ -43,12 +48,13 @@ def test_full_size_sampled_units(name):
         assert_scores_close(got_s, pooled, f"{name} unit {(l, b, h)}")
         ora_idx = oracle.select_unit(pooled.astype(np.float32), wl.L, wl.w, m)
         gk = hp.kept[l, b, h].cpu().numpy()
-        nd = assert_kept_match(gk, ora_idx, pooled, wl.L, wl.w, m, f"{name} unit {(l, b, h)}")
-        if nd:
-            continue
+        assert_kept_match(gk, ora_idx, pooled, wl.L, wl.w, m, f"{name} unit {(l, b, h)}")
+        # Compaction and decode follow the GPU's own kept set: equal to the oracle's, or a
+        # selection that differs only inside the tie band and is just as valid.
+        idx = gk[:m]
         Kc = np.zeros((wl.L_cap, wl.d), np.float32)
         Vc = np.zeros((wl.L_cap, wl.d), np.float32)
-        Kc[:m], Vc[:m] = oracle.gather_unit(K0, ora_idx), oracle.gather_unit(V0, ora_idx)
+        Kc[:m], Vc[:m] = oracle.gather_unit(K0, idx), oracle.gather_unit(V0, idx)
         dk = np32(hp.dk[:, l, b, h])
         dv = np32(hp.dv[:, l, b, h])
         Kc[m:m + wl.decode_steps], Vc[m:m + wl.decode_steps] = dk, dv
@@ -60,7 +66,9 @@ def test_full_size_sampled_units(name):
             got = hp.out[s, l, b, h * G:(h + 1) * G].float().cpu().numpy()
             for g in range(G):
                 o, lse = oracle.decode_unit(qs[g], Kc, Vc, m + s + 1, wl.scale())
-                assert (np.abs(got[g] - o) <= DECODE_ATOL[wl.dtype]).all(), (name, s, l, b, h, g)
+                # a bf16 output adds its own rounding: half an ulp, at most 2^-8 of |o|
+                tol = atol + (np.abs(o) * 2.0 ** -8 if out_dtype == torch.bfloat16 else 0.0)
+                assert (np.abs(got[g] - o) <= tol).all(), (name, s, l, b, h, g, float(np.abs(got[g] - o).max()))
                 assert abs(float(hp.lse[s, l, b, h * G + g]) - lse) < 1e-3
     if hp.has_vocab:
         # the penalty ran once per decode step on the same logits buffer

@@ -2,7 +2,9 @@
 
 The oracle ranks its own float64 scores (rounded to float32, the precision the
 kernel decides in); kept sets must agree except near-boundary candidates (see
-helpers).  Decode outputs are compared on every unit whose kept set agrees."""
+helpers).  Decode outputs are compared on every unit against the oracle's attention
+over the rows the GPU kept: the oracle's own set, or one that differs from it only
+inside the tie band and is just as valid a selection."""
 import numpy as np
 import pytest
 import torch
@@ -51,8 +53,8 @@ def run_pipeline(wl, ratio=None, steps=None):
                 np.testing.assert_array_equal(Kg[l, b, h, :m], K0[l, b, h, gi])  # compaction is exact
                 np.testing.assert_array_equal(Vg[l, b, h, :m], V0[l, b, h, gi])
                 same[l, b, h] = nd == 0
-                Kc[l, b, h, :m] = oracle.gather_unit(K0[l, b, h], ora_idx[l, b, h, :m])
-                Vc[l, b, h, :m] = oracle.gather_unit(V0[l, b, h], ora_idx[l, b, h, :m])
+                Kc[l, b, h, :m] = oracle.gather_unit(K0[l, b, h], gi)
+                Vc[l, b, h, :m] = oracle.gather_unit(V0[l, b, h], gi)
     assert same.mean() >= 0.9, f"kept sets differ (within the tie band) on {(~same).sum()} units"
     L_np = np.broadcast_to(keep.reshape(1, -1, 1), lens_np.shape).copy()
     np.testing.assert_array_equal(lens.cpu().numpy(), L_np)
@@ -69,8 +71,6 @@ def run_pipeline(wl, ratio=None, steps=None):
                     Lc = L_np[l, b, h]
                     Kc[l, b, h, Lc], Vc[l, b, h, Lc] = kn_np[l, b, h], vn_np[l, b, h]
                     L_np[l, b, h] = Lc + 1
-                    if not same[l, b, h]:
-                        continue
                     for g in range(G):
                         o, _ = oracle.decode_unit(q_np[l, b, h * G + g], Kc[l, b, h], Vc[l, b, h], Lc + 1,
                                                   wl.scale())

@@ -1,4 +1,5 @@
-"""reco_select_compact vs the oracle: kept indices and compacted rows bit-exact.
+"""reco_select_compact (and its two halves as separate calls, reco_select_topm then
+reco_compact) vs the oracle: kept indices and compacted rows bit-exact.
 
 The scores are generator inputs given to both sides, so the selection decision is
 taken on identical float32 values and must agree exactly, ties included."""
@@ -7,7 +8,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import gpu_select, np32
+from helpers import gpu_select, gpu_select_split, np32
 from paper_2608_04771_gb300 import reco
 from paper_2608_04771_gb300 import workloads as W
 
@@ -26,12 +27,12 @@ def _bits(t: torch.Tensor) -> np.ndarray:
     return t.cpu().view(torch.int16 if t.dtype == torch.bfloat16 else torch.int32).numpy()
 
 
-def _run_case(wl, lens_np, keep_np, scores_np, seed=0):
+def _run_case(wl, lens_np, keep_np, scores_np, split=False):
     K, V = W.make_cache(wl, DEV, canary=False)
     K0, V0 = K.clone(), V.clone()
     lens = torch.from_numpy(lens_np).to(DEV)
     scores = torch.from_numpy(scores_np).to(DEV)
-    kept = gpu_select(wl, K, V, scores, lens, keep_np)
+    kept = (gpu_select_split if split else gpu_select)(wl, K, V, scores, lens, keep_np)
     reco.reco_check()
     ora_idx = oracle.select_batch(scores_np, lens_np, keep_np, wl.w)
     Kb, Vb, K0b, V0b = _bits(K), _bits(V), _bits(K0), _bits(V0)
@@ -54,8 +55,9 @@ def _tie_scores(rng, shape, levels):
     return (rng.integers(0, levels, shape) / levels).astype(np.float32)
 
 
+@pytest.mark.parametrize("split", [False, True])
 @pytest.mark.parametrize("dtype,d", [("bf16", 128), ("bf16", 64), ("f32", 64), ("f32", 128)])
-def test_select_compact_ragged_with_ties(dtype, d):
+def test_select_compact_ragged_with_ties(dtype, d, split):
     wl = W.WORKLOADS["1.5b"].reduced(layers=2, batch=3, h_q=4, h_kv=2, d=d, dtype=dtype, L=1200,
                                      decode_steps=37, w=32, outliers=0)
     rng = np.random.default_rng(1)
@@ -65,10 +67,11 @@ def test_select_compact_ragged_with_ties(dtype, d):
     scores = rng.random((wl.layers, wl.batch, wl.h_kv, wl.L_cap)).astype(np.float32)
     scores[0, 1] = _tie_scores(rng, wl.L_cap, 7)  # heavy ties
     scores[1, 2, 0] = 0.5  # all equal: lowest indices win
-    _run_case(wl, lens, keep, scores)
+    _run_case(wl, lens, keep, scores, split)
 
 
-def test_select_edge_cases():
+@pytest.mark.parametrize("split", [False, True])
+def test_select_edge_cases(split):
     wl = W.WORKLOADS["7b"].reduced(layers=1, batch=5, h_q=4, h_kv=1, L=300, decode_steps=0, w=16)
     rng = np.random.default_rng(2)
     lens = np.array([[[300]], [[300]], [[16]], [[300]], [[257]]], np.int32).reshape(1, 5, 1)
@@ -76,7 +79,7 @@ def test_select_edge_cases():
     scores = rng.random((1, 5, 1, 300)).astype(np.float32)
     scores[0, 3, 0, :] = 1.0
     scores[0, 3, 0, 0] = 0.0  # drop only candidate 0: every kept row moves up by one (in-place chain)
-    _run_case(wl, lens, keep, scores)
+    _run_case(wl, lens, keep, scores, split)
 
 
 def test_select_plateaus_from_maxpool_shape():
@@ -115,3 +118,56 @@ def test_select_compact_beyond_shared_memory_keys():
     lens = np.array([[[50_000], [49_500]]], np.int32)
     keep = np.array([12_345, 30_001], np.int32)
     _run_case(wl, lens, keep, _tie_scores(rng, (1, 2, 1, wl.L_cap), 4096))
+
+
+def test_select_topm_touches_only_the_indices():
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=3, h_q=8, h_kv=2, L=700, decode_steps=5, w=32)
+    K, V = W.make_cache(wl, DEV, canary=False)
+    K0, V0 = K.clone(), V.clone()
+    rng = np.random.default_rng(8)
+    lens_np = rng.integers(400, 701, (2, 3, 2)).astype(np.int32)
+    keep_np = np.array([100, 32, 399], np.int32)
+    scores_np = rng.random((2, 3, 2, wl.L_cap)).astype(np.float32)
+    lens = torch.from_numpy(lens_np).to(DEV)
+    kv = reco.make_kv(K, V, wl.h_q)
+    kept = torch.full(K.shape[:4], -1, dtype=torch.int32, device=DEV)
+    ws = reco.workspace(reco.RECO_OP_SELECT, kv, wl.w, DEV)
+    reco.reco_select_topm(kv, torch.from_numpy(scores_np).to(DEV), lens, torch.from_numpy(keep_np).to(DEV), wl.w,
+                          kept, ws)
+    reco.reco_check()
+    assert torch.equal(K.view(torch.int16), K0.view(torch.int16)) and torch.equal(V.view(torch.int16),
+                                                                                   V0.view(torch.int16))
+    np.testing.assert_array_equal(lens.cpu().numpy(), lens_np)
+    ora = oracle.select_batch(scores_np, lens_np, keep_np, wl.w)
+    got = kept.cpu().numpy()
+    for l in range(2):
+        for b in range(3):
+            for h in range(2):
+                m = int(keep_np[b])
+                np.testing.assert_array_equal(got[l, b, h, :m], ora[l, b, h, :m])
+                assert (got[l, b, h, m:] == -1).all()
+
+
+def test_compact_refuses_indices_outside_r_to_L():
+    """reco_compact copies only sources in [r, L): a source below its destination (which an
+    earlier destination may have overwritten) or at/after the unit's length is refused."""
+    wl = W.WORKLOADS["7b"].reduced(layers=1, batch=2, h_q=4, h_kv=1, L=64, decode_steps=4, w=4)
+    K, V = W.make_cache(wl, DEV, canary=False)
+    K0 = K.clone()
+    kv = reco.make_kv(K, V, wl.h_q)
+    lens = torch.tensor([[[64], [40]]], dtype=torch.int32, device=DEV)
+    keep = torch.tensor([8, 8], dtype=torch.int32, device=DEV)
+    kept = torch.zeros(K.shape[:4], dtype=torch.int32, device=DEV)
+    kept[0, 0, 0, :8] = torch.tensor([2, 0, 9, 20, 60, 61, 62, 63])  # row 1 <- row 0: refused
+    kept[0, 1, 0, :8] = torch.tensor([1, 2, 3, 4, 5, 6, 7, 40])  # row 40 == L: refused
+    reco.reco_compact(kv, kept, lens, keep, wl.w)
+    with pytest.raises(reco.RecoError) as e:
+        reco.reco_check()
+    assert e.value.status == reco.RECO_EDEVICE
+    Kb, K0b = _bits(K), _bits(K0)
+    for r, src in enumerate([2, None, 9, 20, 60, 61, 62, 63]):
+        np.testing.assert_array_equal(Kb[0, 0, 0, r], K0b[0, 0, 0, r if src is None else src])
+    for r, src in enumerate([1, 2, 3, 4, 5, 6, 7, None]):
+        np.testing.assert_array_equal(Kb[0, 1, 0, r], K0b[0, 1, 0, r if src is None else src])
+    assert lens.flatten().tolist() == [8, 8]
+    reco.reco_check()

@@ -50,6 +50,11 @@ class OracleReplay:
         self.diverged = set()  # (seq, layer, kv head) whose kept set differed within the tie band
         self.expected_probes = set()
         self.sampled = 0  # draws checked
+        # cache bytes held after every token, from the replay's own lengths (Table 3's
+        # memory, cache only): K and V rows of every layer and KV head of the active sequences
+        self.row_bytes = 2 * wl.layers * wl.h_kv * wl.d * wl.elem_bytes
+        self.peak_bytes = 0
+        self.byte_tokens = 0
 
     def on_token(self, t, tr, out, lse, logits):
         wl = self.wl
@@ -63,6 +68,13 @@ class OracleReplay:
             self.K[:, s, :, L] = kn[:, s]
             self.V[:, s, :, L] = vn[:, s]
             self.lens[s] = L + 1
+        held = sum(self.lens[s] for s in act) * self.row_bytes
+        self.peak_bytes = max(self.peak_bytes, held)
+        self.byte_tokens += held
+        # the device's lengths after the decode's append are the replay's, on every layer and head
+        dev_lens = tr.lens_dev.cpu().numpy()
+        for i, s in zip(pos, act):
+            assert (dev_lens[:, i, :] == self.lens[s]).all(), (t, s, self.lens[s])
         if t % self.decode_every == 0:
             lens = np.array([[[self.lens[s]] * wl.h_kv for s in act]] * wl.layers, np.int32)
             o_ref, lse_ref = oracle.decode_batch(q[:, act], self.K[:, act], self.V[:, act], lens, wl.scale())
@@ -139,6 +151,9 @@ def _run(spec, track=None, decode_every=1, use_graph=False, input_pool=0):
         p_ref, stop_ref = oracle.answer_ppl(np32(z), tok.cpu().numpy(), None, spec.base.tau_p)
         assert abs(ppl - p_ref[0]) <= PPL_RTOL * p_ref[0]
         assert stopped == bool(stop_ref[0])
+    if track is None:  # every sequence followed: the trace's cache-bytes counters are the replay's
+        assert ev.peak_cache_bytes == rep.peak_bytes > 0
+        assert ev.cache_byte_tokens == rep.byte_tokens
     return tr, rep, ev
 
 
@@ -164,7 +179,7 @@ def test_trace_interval_trigger():
     tr, rep, ev = _run(spec)
     assert rep.tie_diffs == 0
     assert 0 < ev.compressions < ev.steps_completed  # some boundaries skip compression
-    assert ev.peak_cache_bytes > 0 and ev.generated > 0
+    assert ev.generated > 0
 
 
 def test_trace_reading_B_reduced_with_stops():
@@ -187,3 +202,17 @@ def test_trace_full_size_sampled():
     # near-tie flips (fp32 vs fp64 scores within 1e-5 of the cut) stop the comparison of that unit only
     assert len(rep.diverged) <= 0.05 * 2 * spec.base.layers * spec.base.h_kv, rep.diverged
     assert ev.lse_scorings > 10 * ev.two_pass_scorings  # steps are Poisson(96)+16 >> w tokens
+
+
+def test_trace_cache_bytes_without_compression():
+    """With compression switched off by the interval trigger (S larger than any growth) the
+    cache holds every token: the peak is the closed form B * (prompt + generated) rows and the
+    per-token sum is B * sum_t (prompt + t + 1) rows."""
+    base = W.WORKLOADS["7b"].reduced(layers=1, vocab=2000, tau_h=1.5)  # no probe: every sequence runs on
+    spec = trace.TraceSpec(base, batch=3, prompt=64, generated=150, step_mean=30, step_min=8, seed=7,
+                           reading="A", interval=10_000)
+    tr, rep, ev = _run(spec, decode_every=50)
+    assert ev.compressions == 0
+    row = 2 * base.layers * base.h_kv * base.d * base.elem_bytes
+    assert ev.peak_cache_bytes == 3 * (64 + 150) * row
+    assert ev.cache_byte_tokens == 3 * sum(64 + t + 1 for t in range(150)) * row

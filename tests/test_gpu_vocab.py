@@ -83,6 +83,18 @@ def test_ppl_ragged_lengths_odd_vocab_and_empty():
     _ppl_case(z, tok, [9, 1, 0, 4, 20])
 
 
+def test_ppl_logits_not_16_byte_aligned():
+    """V a multiple of 4 but the logits one float into their allocation: the kernel must
+    not take its 16-byte vector loads (a misaligned vector load faults)."""
+    rng = np.random.default_rng(5)
+    B, n, V = 3, 7, 2048
+    buf = torch.from_numpy((rng.standard_normal(B * n * V + 1) * 2).astype(np.float32)).to(DEV)
+    z = buf[1:].view(B, n, V)
+    assert z.data_ptr() % 16 == 4 and z.is_contiguous()
+    tok = torch.from_numpy(rng.integers(0, V, (B, n)).astype(np.int32)).to(DEV)
+    _ppl_case(z, tok, [7, 2, 5])
+
+
 def test_ppl_golden_two_token():
     z = torch.tensor([[[0.0] * 8, [float(np.log(7.0))] + [0.0] * 7]], device=DEV)
     tok = torch.tensor([[5, 0]], dtype=torch.int32, device=DEV)

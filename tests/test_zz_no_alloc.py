@@ -50,6 +50,25 @@ def test_static_matches_workspace_entry_point_twice():
     _both(z2, tok2, [40, 3, 0, 17, 40])
 
 
+def test_static_allocates_no_device_memory():
+    """The defining property: no device memory is taken by the calls themselves.
+    Inputs, outputs and a first call (which loads the kernels) come before the count."""
+    wl = W.WORKLOADS["7b"].reduced(vocab=30000)
+    z, tok = W.make_answer(wl, DEV)
+    B = z.shape[0]
+    ppl, stop = torch.empty(B, device=DEV), torch.empty(B, dtype=torch.uint8, device=DEV)
+    reco.reco_answer_ppl_static(z, tok, None, 1.1, ppl, stop)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    reserved0 = torch.cuda.memory_reserved()
+    for _ in range(2):
+        reco.reco_answer_ppl_static(z, tok, None, 1.1, ppl, stop)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0 and torch.cuda.memory_reserved() == reserved0
+    reco.reco_check()
+
+
 def test_static_rejects_more_rows_than_its_array():
     n = reco.RECO_PPL_STATIC_MAX_ROWS // 4 + 1
     z = torch.zeros((4, n, 4), device=DEV)
@@ -59,3 +78,15 @@ def test_static_rejects_more_rows_than_its_array():
     with pytest.raises(reco.RecoError) as e:
         reco.reco_answer_ppl_static(z, tok, None, 1.1, ppl, stop)
     assert e.value.status == reco.RECO_EINVAL and "static scratch" in str(e.value)
+    # the grid limits of the workspace entry point hold here too: same inputs, same status
+    for B, n in ((65536, 1), (70000, 0)):
+        z = torch.zeros((B, n, 4), device=DEV)
+        tok = torch.zeros((B, n), dtype=torch.int32, device=DEV)
+        ppl = torch.empty(B, device=DEV)
+        stop = torch.empty(B, dtype=torch.uint8, device=DEV)
+        ws = reco.workspace(reco.RECO_OP_PPL, None, B * n, DEV)
+        with pytest.raises(reco.RecoError) as e1:
+            reco.reco_answer_ppl(z, tok, None, 1.1, ppl, stop, ws)
+        with pytest.raises(reco.RecoError) as e2:
+            reco.reco_answer_ppl_static(z, tok, None, 1.1, ppl, stop)
+        assert e1.value.status == e2.value.status == reco.RECO_EUNSUPPORTED
