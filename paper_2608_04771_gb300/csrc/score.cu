@@ -30,8 +30,10 @@ ScoreWs score_ws_layout(const reco_kv &kv, int w, void *base)
         return r;
     };
     ScoreWs ws;
-    ws.part_m = (float *)take(units * nch * R * 4);
-    ws.part_z = (float *)take(units * nch * R * 4);
+    // up to two partials per (unit, chunk, row): the tensor-core pass 1 may split a
+    // chunk's key tiles between two epilogue groups
+    ws.part_m = (float *)take(units * nch * 2 * R * 4);
+    ws.part_z = (float *)take(units * nch * 2 * R * 4);
     ws.rowb = (float *)take(units * R * 4);
     ws.raw = (float *)take(units * (size_t)kv.L_cap * 4);
     ws.ulist = (int32_t *)take(units * 4);
@@ -111,10 +113,11 @@ __global__ void __launch_bounds__(256) score_rowstats_simt(
     }
 }
 
-// Merge the chunk partials of each row into b_r = m_r + log2(Z_r).
+// Merge the partials of each row (per_chunk of them for each key chunk, laid out
+// [unit][chunk][per_chunk][R]) into b_r = m_r + log2(Z_r).
 __global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap, int R,
-                              int n_chunks, const float *__restrict__ part_m, const float *__restrict__ part_z,
-                              float *__restrict__ rowb, long units)
+                              int n_chunks, int per_chunk, const float *__restrict__ part_m,
+                              const float *__restrict__ part_z, float *__restrict__ rowb, long units)
 {
     long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= units * R) return;
@@ -122,10 +125,10 @@ __global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, 
     int r = (int)(i % R);
     int L = lens[u];
     if (L < w || L > L_cap || mask.skip(u, L, w, L_cap)) return;
-    int used = (L + kScoreChunk - 1) / kScoreChunk;
+    int used = ((L + kScoreChunk - 1) / kScoreChunk) * per_chunk;
     float m = -INFINITY, z = 0.f;
     for (int c = 0; c < used; ++c) {
-        size_t o = ((size_t)u * n_chunks + c) * R + r;
+        size_t o = ((size_t)u * n_chunks * per_chunk + c) * R + r;
         lse_merge(m, z, part_m[o], part_z[o]);
     }
     rowb[i] = m + log2f(z);
@@ -322,6 +325,7 @@ cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const in
 cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
                                   float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
 bool score_tc_supported(const reco_kv &kv, int w);
+int score_tc_pass1_groups(int R);
 
 // SIMT passes; with pass1 false the row normalisers are already in ws.rowb.
 template <typename T, int D>
@@ -340,7 +344,7 @@ static cudaError_t score_simt(const reco_kv &kv, const T *q_win, const int32_t *
                                                     nch, c2, ws.part_m, ws.part_z, err);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         long n = units * R;
-        score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch, ws.part_m,
+        score_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch, 1, ws.part_m,
                                                                   ws.part_z, ws.rowb, units);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
@@ -394,8 +398,8 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
         if (used_tc) {
             const int R = (kv.H_q / kv.H_kv) * w;
             const int nch = (kv.L_cap + kScoreChunk - 1) / kScoreChunk;
-            score_combine<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, nch,
-                                                                              ws.part_m, ws.part_z, ws.rowb, units);
+            score_combine<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(
+                lens, mask, w, kv.L_cap, R, nch, score_tc_pass1_groups(R), ws.part_m, ws.part_z, ws.rowb, units);
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
             bool used2 = false;
             e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used2);

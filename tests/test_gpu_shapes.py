@@ -27,8 +27,10 @@ CASES = {
     "g8_r256": dict(h_q=16, h_kv=2, w=32, L=1300),         # tensor decode at G = 8; pass 2 N = 256
     "g16_simt_decode": dict(h_q=16, h_kv=1, w=16, L=800),  # G = 16: bf16 decode on the SIMT path
     "w1_pool1": dict(w=1, pool=1, L=600),                  # one window query, Eq. 2 without pooling
-    "r320_pool9": dict(h_q=10, h_kv=2, w=64, pool=9, L=1500),  # split-column pass 2
-    "r384_max": dict(h_q=12, h_kv=2, w=64, L=1000),        # largest tensor-core window
+    "r320_pool9": dict(h_q=10, h_kv=2, w=64, pool=9, L=1500),  # 32B-class window: 3 query tiles, 4 x 80 columns
+    "r384": dict(h_q=12, h_kv=2, w=64, L=1000),            # 3 query tiles, full
+    "r448_7b_heads_w64": dict(w=64, L=1200),               # G = 7 with w = 64: 4 query tiles, 4 x 112 columns
+    "r512_max": dict(h_q=8, h_kv=1, w=64, L=1000),         # largest tensor-core window
     "fp32_d128": dict(dtype="f32", d=128, L=600),
 }
 
@@ -40,7 +42,7 @@ def test_pipeline_shape(name):
 
 
 def test_window_rows_beyond_both_scoring_paths_are_rejected():
-    wl = BASE.reduced(layers=1, batch=1, h_q=8, h_kv=1, w=64, L=300, decode_steps=0)  # G*w = 512
+    wl = BASE.reduced(layers=1, batch=1, h_q=8, h_kv=1, w=66, L=300, decode_steps=0)  # G*w = 528
     K, V = W.make_cache(wl, "cuda", canary=False)
     kv = reco.make_kv(K, V, wl.h_q)
     st = reco.lib().reco_score_cache(ctypes.byref(kv), ctypes.c_void_p(K.data_ptr()), ctypes.c_void_p(16),
