@@ -663,8 +663,11 @@ def run_e2e(hp, wl, args, world):
             if timed:
                 c0 = torch.cuda.Event(enable_timing=True)
                 c0.record(cps)
-            for k, h in host.items():
-                getattr(s, k).copy_(h, non_blocking=True)
+            for k, h in host.items():  # in copies of at most 1 GiB each
+                dst = getattr(s, k).view(-1).view(torch.uint8)
+                src = h.view(-1).view(torch.uint8)
+                for o in range(0, src.numel(), 1 << 30):
+                    dst[o:o + (1 << 30)].copy_(src[o:o + (1 << 30)], non_blocking=True)
             ready[i % 2].record(cps)
             if timed:
                 c1 = torch.cuda.Event(enable_timing=True)
@@ -698,8 +701,8 @@ def run_e2e(hp, wl, args, world):
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n,
             "h2d_GBps": h2d / cp_ms / 1e6, "h2d_ms_per_step": cp_ms,
             "pinned_near_gpu": bool(local),
-            "schedule": "two device buffer sets and three streams: step i+1's host-to-device copies and step "
-                        "i-1's read-back overlap step i's compute"}
+            "schedule": "two device buffer sets and three streams: step i+1's host-to-device copies (in copies of "
+                        "at most 1 GiB) and step i-1's read-back overlap step i's compute"}
 
 
 def run_trace(args):
@@ -740,8 +743,8 @@ def run_trace(args):
                    "window": "Eq. 2's window queries are the last w decoded tokens' queries; a boundary scores "
                              "in one pass with their decode lse (kept in a device ring) when none of the "
                              "compressing sequences was compressed within the window, else in two passes",
-                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode + penalty and draw "
-                                       "+ lse ring push)" if use_graph else "direct calls"},
+                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode writing its lse "
+                                       "into the ring + penalty and draw)" if use_graph else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),
                   "boundary_scorings": {"one_pass_decode_lse": ev.lse_scorings, "two_pass": ev.two_pass_scorings},

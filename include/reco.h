@@ -236,6 +236,21 @@ reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new
                              int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
                              void *ws, size_t ws_bytes, cudaStream_t stream);
 
+/* reco_decode_attn whose log-sum-exps go into the device ring that
+ * reco_score_cache_lse reads (Sec. 3.2's observation window: the lse of the last
+ * decoded tokens are the row normalisers of Eq. 2), instead of an lse array: the launch
+ * writes lse[layer,b,hq] into rows *slot and *slot + slots of ring and then advances
+ * *slot to (*slot + 1) % slots, all on the device, so a captured graph decodes every
+ * token with no separate push.  It is reco_decode_attn followed by reco_lse_push in one
+ * launch, with the same results.
+ *   ring : [2 * slots][n_layers * B * H_q] float32 (device, two rows written)
+ *   slot : int64 (device, read and advanced); a value outside [0, slots) writes no ring
+ *          row, leaves *slot as it is and sets the device error word
+ * Every other argument, the result and the workspace are those of reco_decode_attn.    */
+reco_status reco_decode_attn_ring(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,
+                                  int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *ring,
+                                  int slots, int64_t *slot, void *ws, size_t ws_bytes, cudaStream_t stream);
+
 /* Eq. 3 + Eq. 4 (Sec. 3.3, reward-banded reflection penalty), in place:
  *   beta_b = 0, beta/2 or beta by the band of rewards[b] (float32 compares);
  *   logits[b, u] -= beta_b once for each distinct id u in ids[0..n_ids-1];

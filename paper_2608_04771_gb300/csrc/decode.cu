@@ -62,7 +62,34 @@ struct DecodeArgs {
     int units, Hq, Hkv, G, L_cap, append, out_bf16;
     float c2;  // scale * log2(e)
     unsigned *err;
+    float *ring;      // or nullptr: lse rows ring[*slot] and ring[*slot + slots], each [nq]
+    long long *slot;  // device ring row, advanced by one (mod slots) per launch
+    int slots;
+    long long nq;     // query heads of the launch (layers * B * H_q)
 };
+
+// The ring row this launch writes (read once the previous kernel's writes are visible),
+// or -1 without a ring; a slot outside [0, slots) writes nothing and sets the error word.
+__device__ __forceinline__ long long ring_row(const DecodeArgs &a)
+{
+    if (!a.ring) return -1;
+    const long long s = *a.slot;
+    if (s < 0 || s >= a.slots) {
+        raise_error(a.err, ERR_INTERNAL);
+        return -1;
+    }
+    return s;
+}
+
+// lse of query row i: to the lse output and, with a ring, to ring rows rs and rs + slots.
+__device__ __forceinline__ void put_lse(const DecodeArgs &a, long long rs, size_t i, float v)
+{
+    if (a.lse) a.lse[i] = v;
+    if (rs >= 0) {
+        a.ring[rs * a.nq + (long long)i] = v;
+        a.ring[(rs + a.slots) * a.nq + (long long)i] = v;
+    }
+}
 
 // atomicAdd with acquire-release semantics at GPU scope.
 __device__ __forceinline__ int atom_add_acq_rel(int *p, int v)
@@ -95,6 +122,7 @@ __global__ void __launch_bounds__(128) decode_simt(DecodeArgs a)
     const long u = blockIdx.x;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const int L = a.lens[u];
+    const long long rs = ring_row(a);
     const bool ok = unit_ok(L, a.L_cap, a.append);
     if (!ok && threadIdx.x == 0) raise_error(a.err, (a.append && L == a.L_cap) ? ERR_ROOM : ERR_LEN);
     const int Le = ok ? L + a.append : 0;
@@ -169,7 +197,7 @@ __global__ void __launch_bounds__(128) decode_simt(DecodeArgs a)
         }
         const size_t row = (size_t)(lb * a.Hq + (long)h * G + g);
         store_out<T>(a.out, a.out_bf16, row * D + dd, Ls > 0.f ? O / Ls : 0.f);
-        if (dd == 0 && a.lse) a.lse[row] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+        if (dd == 0) put_lse(a, rs, row, Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY);
     }
     if (ok && a.append) {
         for (int e = threadIdx.x; e < D; e += blockDim.x) {
@@ -267,6 +295,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
     __syncwarp();
     wait_prior_grid();  // lens, q and the new rows may come from the previous kernels
+    const long long rs = ring_row(a);  // the ring row this launch writes (-1: none)
 
     // ---- plan: identical in every CTA (lens are not modified until every warp is done).
     // Each unit's keys form nb_u = ceil(le_u / 16) blocks; the blocks of all units are laid
@@ -662,7 +691,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                     }
                 }
             }
-            if (c == 0 && g < G && a.lse) a.lse[qrow0 + g] = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
+            if (c == 0 && g < G) put_lse(a, rs, qrow0 + g, l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY);
         } else {
             float *po = a.part_o + (size_t)item * G * D;
 #pragma unroll
@@ -748,8 +777,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                         for (int e = 0; e < PER; ++e)
                             store_out<__nv_bfloat16>(a.out, out_bf16, (qrow0 + qq) * D + lane * PER + e,
                                                      acc[qq][e] * inv);
-                        if (lane == 0 && a.lse)
-                            a.lse[qrow0 + qq] = Lq[qq] > 0.f ? (Mq[qq] + log2f(Lq[qq])) * kLn2 : -INFINITY;
+                        if (lane == 0)
+                            put_lse(a, rs, qrow0 + qq, Lq[qq] > 0.f ? (Mq[qq] + log2f(Lq[qq])) * kLn2 : -INFINITY);
                     }
                 }
             }
@@ -804,8 +833,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         if (lane == 0) {
             a.counters[0] = 0;
             a.counters[1] = 0;
+            if (rs >= 0) *a.slot = (rs + 1) % a.slots;  // every warp has read the row by now
         }
     }
+}
+
+// The ring slot's advance after the SIMT decode (its CTAs have no last-warp step).
+__global__ void ring_advance(long long *slot, int slots)
+{
+    const long long s = *slot;
+    if (s >= 0 && s < slots) *slot = (s + 1) % slots;
 }
 
 // ---------------------------------------------------------------- host side
@@ -817,7 +854,8 @@ static bool encode_cache_map(CUtensorMap *map, const void *base, unsigned long l
 
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
                           int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
-                          const DecodeWs &ws, unsigned *err, cudaStream_t s)
+                          const DecodeWs &ws, unsigned *err, cudaStream_t s, float *ring, int slots,
+                          long long *slot)
 {
     DecodeArgs a;
     a.K = kv.k;
@@ -840,6 +878,10 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.out_bf16 = out_dtype == RECO_BF16 ? 1 : 0;
     a.c2 = scale * kLog2e;
     a.err = err;
+    a.ring = ring;
+    a.slot = slot;
+    a.slots = slots;
+    a.nq = (long long)kv.n_layers * kv.B * kv.H_q;
     const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
     // partial slots: two per warp of the grid
     const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.part_slots;
@@ -868,6 +910,9 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
         if (kv.d == 64) decode_simt<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
         else decode_simt<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
     }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || !ring) return e;
+    ring_advance<<<1, 1, 0, s>>>(slot, slots);
     return cudaGetLastError();
 }
 

@@ -78,9 +78,12 @@ cudaError_t launch_select_only(const reco_kv &kv, const float *scores, const int
                                int w, int32_t *kept_idx, const SelectWs &ws, unsigned *err, cudaStream_t s);
 cudaError_t launch_compact(const reco_kv &kv, const int32_t *kept_idx, int32_t *lens, const int32_t *keep, int w,
                            unsigned *err, cudaStream_t s);
+// ring: optional [2 * slots][layers * B * H_q] lse ring; the launch writes rows *slot and
+// *slot + slots and advances *slot.
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
                           int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
-                          const DecodeWs &ws, unsigned *err, cudaStream_t s);
+                          const DecodeWs &ws, unsigned *err, cudaStream_t s, float *ring = nullptr,
+                          int slots = 0, long long *slot = nullptr);
 cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
                            const float *rewards, float tau_l, float tau_h, float beta, float *beta_out,
                            unsigned *err, cudaStream_t s);

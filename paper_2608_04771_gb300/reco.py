@@ -21,7 +21,7 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = ran
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
            "reco_score_cache_lse", "reco_lse_push", "reco_select_compact", "reco_select_topm", "reco_compact",
-           "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
+           "reco_decode_attn", "reco_decode_attn_ring", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
            "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
 
@@ -70,6 +70,7 @@ def lib():
     L.reco_select_topm.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_compact.argtypes = [kvp, vp, vp, vp, i32, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
+    L.reco_decode_attn_ring.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, i32, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
     L.reco_penalty_sample.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp]
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
@@ -77,7 +78,8 @@ def lib():
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
                  "reco_score_cache", "reco_score_cache_lse", "reco_lse_push", "reco_select_compact",
                  "reco_select_topm", "reco_compact",
-                 "reco_decode_attn", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
+                 "reco_decode_attn", "reco_decode_attn_ring", "reco_reflect_penalty", "reco_penalty_sample",
+                 "reco_answer_ppl",
                  "reco_answer_ppl_static"):
         getattr(L, name).restype = i32
     _lib = L
@@ -209,6 +211,16 @@ def reco_decode_attn(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, lse,
     _ok(lib().reco_decode_attn(ctypes.byref(kv), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(lens),
                                float(scale), _ptr(out), _dtype_code(out.dtype), _ptr(lse), _ptr(ws),
                                ws.numel(), _stream(stream)))
+
+
+def reco_decode_attn_ring(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, ring, slot, ws, stream=None):
+    """reco_decode_attn with the lse written into ring rows slot and slot + S (ring [2 * S, n]
+    float32) and slot (one-element int64 device tensor) advanced, on the device."""
+    if ring.dim() < 2 or ring.shape[0] % 2:
+        raise ValueError("ring must have an even number of rows")
+    _ok(lib().reco_decode_attn_ring(ctypes.byref(kv), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(lens), float(scale),
+                                    _ptr(out), _dtype_code(out.dtype), _ptr(ring), int(ring.shape[0]) // 2,
+                                    _ptr(slot), _ptr(ws), ws.numel(), _stream(stream)))
 
 
 def reco_reflect_penalty(logits, ids, rewards, tau_l=0.4, tau_h=0.8, beta=4.0, beta_out=None,

@@ -192,7 +192,6 @@ class Trace:
         self.lse_ring = torch.zeros((2 * self.R, wl.layers, spec.batch, wl.h_q), dtype=torch.float32,
                                     device=device)
         self.slot_dev = torch.zeros(1, dtype=torch.long, device=device)
-        self._side = torch.cuda.Stream(device=device) if use_graph else None  # graph branch of the ring push
         self._slot_t = -1  # the token whose ring slot slot_dev holds
         self.since = [0] * spec.batch
         self._rebuild()
@@ -368,19 +367,13 @@ class Trace:
                 # fewer nanoseconds than 8-byte ones for the same bytes
                 torch.index_select(self._apool.view(torch.complex128), 0, self.slot_dev,
                                    out=self.g_in.view(torch.complex128).view(1, -1))
-            reco.reco_decode_attn(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
-                                  self.g_lse, self.ws_decode)
-            # the token's lse into the ring, which advances the slot (the next token's pool
-            # slot): a branch of the graph beside the penalty and draw, joined at its end
-            main = torch.cuda.current_stream()
-            fork = torch.cuda.Event()
-            fork.record(main)
-            self._side.wait_event(fork)
-            reco.reco_lse_push(self.g_lse, self.lse_ring, self.slot_dev, stream=self._side)
+            # the token's lse goes straight into the ring, and the decode advances the slot
+            # (the next token's pool slot)
+            reco.reco_decode_attn_ring(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
+                                       self.lse_ring, self.slot_dev, self.ws_decode)
             if self.g_logits is not None:
                 reco.reco_penalty_sample(self.g_logits, self.ids, self.g_rw, self.g_u, self.g_tok, self.ws_sample,
                                          wl.tau_l, wl.tau_h, wl.beta)
-            main.wait_stream(self._side)
         self.slot_dev.fill_(t % self.R)
         self._slot_t = t
         self.graph = g
@@ -416,12 +409,12 @@ class Trace:
             self.graph.replay()
             self._slot_t = t + 1
             self.tokens = self.g_tok
-            return self.g_out, self.g_lse, self.g_logits
+            return self.g_out, self.lse_ring[t % self.R], self.g_logits
         q, kn, vn = self.active_inputs(t)
         out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
-        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=self.device)
-        reco.reco_decode_attn(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, lse, self.ws_decode)
-        reco.reco_lse_push(lse, self.lse_ring, self.slot_dev)
+        reco.reco_decode_attn_ring(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, self.lse_ring, self.slot_dev,
+                                   self.ws_decode)
+        lse = self.lse_ring[t % self.R]
         self._slot_t = t + 1
         logits = None
         if self.ids is not None:

@@ -183,3 +183,42 @@ def test_lse_push_ring_and_slot():
     with pytest.raises(reco.RecoError):
         reco.reco_check()
     assert torch.equal(ring, before) and int(slot.item()) == 9
+
+
+@pytest.mark.parametrize("dtype,h_q,h_kv,L", [("bf16", 28, 4, 700), ("bf16", 16, 1, 300), ("f32", 8, 2, 200)])
+def test_decode_attn_ring_matches_decode_then_push(dtype, h_q, h_kv, L):
+    """reco_decode_attn_ring is reco_decode_attn followed by reco_lse_push: the same outputs,
+    cache and lengths, the lse in ring rows slot and slot + S (bit-exact), the slot advanced
+    (with a wrap-around), on the TMA path (bf16, G 7), the SIMT path (G 16, and float32)."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=3, h_q=h_q, h_kv=h_kv, L=L, decode_steps=4, dtype=dtype)
+    Ka, Va = W.make_cache(wl, DEV, canary=False)
+    Kb, Vb = Ka.clone(), Va.clone()
+    rng = np.random.default_rng(5)
+    lens_np = rng.integers(1, L + 1, (wl.layers, wl.batch, wl.h_kv)).astype(np.int32)
+    la, lb = torch.from_numpy(lens_np).to(DEV), torch.from_numpy(lens_np).to(DEV)
+    kva, kvb = reco.make_kv(Ka, Va, wl.h_q), reco.make_kv(Kb, Vb, wl.h_q)
+    wsa, wsb = reco.workspace(reco.RECO_OP_DECODE, kva, 0, DEV), reco.workspace(reco.RECO_OP_DECODE, kvb, 0, DEV)
+    S, n = 3, wl.layers * wl.batch * wl.h_q
+    ring_a, ring_b = torch.zeros((2 * S, n), device=DEV), torch.zeros((2 * S, n), device=DEV)
+    slot_a, slot_b = torch.tensor([1], dtype=torch.int64, device=DEV), torch.tensor([1], dtype=torch.int64, device=DEV)
+    for s in range(4):
+        q, kn, vn = W.make_decode_step(wl, s, DEV)
+        oa, ob = torch.empty(q.shape, device=DEV), torch.empty(q.shape, device=DEV)
+        lse = torch.empty(q.shape[:3], device=DEV)
+        reco.reco_decode_attn(kva, q, kn, vn, la, wl.scale(), oa, lse, wsa)
+        reco.reco_lse_push(lse, ring_a, slot_a)
+        reco.reco_decode_attn_ring(kvb, q, kn, vn, lb, wl.scale(), ob, ring_b, slot_b, wsb)
+        reco.reco_check()
+        assert torch.equal(oa, ob) and torch.equal(la, lb)
+        assert torch.equal(ring_a, ring_b) and int(slot_b.item()) == (2 + s) % S
+    assert torch.equal(Ka.view(torch.uint8), Kb.view(torch.uint8))
+    # an out-of-range slot: no ring row written, slot kept, the error word set
+    before = ring_b.clone()
+    slot_b.fill_(S)
+    q, kn, vn = W.make_decode_step(wl, 9, DEV)
+    reco.reco_decode_attn_ring(kvb, q, None, None, lb, wl.scale(), torch.empty(q.shape, device=DEV), ring_b, slot_b, wsb)
+    with pytest.raises(reco.RecoError) as e:
+        reco.reco_check()
+    assert e.value.status == reco.RECO_EDEVICE
+    assert torch.equal(ring_b, before) and int(slot_b.item()) == S
+    reco.reco_check()
