@@ -40,7 +40,8 @@ DecodeWs decode_ws_layout(const reco_kv &kv, void *base)
     };
     DecodeWs ws;
     ws.part_slots = kDecodePartSlots;
-    ws.counters = (int32_t *)take((2 + units) * 4);
+    // merge tickets per unit of the TMA path, which splits a unit of G > 8 heads in two
+    ws.counters = (int32_t *)take((2 + units * (G > 8 ? 2 : 1)) * 4);
     ws.part_ml = (float *)take((size_t)ws.part_slots * G * 2 * 4);
     ws.part_o = (float *)take((size_t)ws.part_slots * G * kv.d * 4);
     ws.bytes = off;
@@ -62,6 +63,7 @@ struct DecodeArgs {
     int units, Hq, Hkv, G, L_cap, append, out_bf16;
     float c2;  // scale * log2(e)
     unsigned *err;
+    int hs, gv;       // TMA path: hs virtual units of gv (<= 8) query heads per unit (G > 8: hs = 2)
     float *ring;      // or nullptr: lse rows ring[*slot] and ring[*slot + slots], each [nq]
     long long *slot;  // device ring row, advanced by one (mod slots) per launch
     int slots;
@@ -307,8 +309,14 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     int *pb = sm_pre;  // [units + 1] prefix of blocks
     const int seg = (units + blockDim.x - 1) / blockDim.x;
     const int u_lo = min(units, tid * seg), u_hi = min(units, u_lo + seg);
+    // Units here are virtual: unit u covers query heads [(u / P) * gv, ...) of the cache
+    // unit u % P (P cache units).  With two halves (G > 8) all first halves come first in
+    // the plan, then all second halves in the same order, so warps w and w + W/2 stream
+    // the same rows at about the same time and the second read mostly hits L2.
+    const int hs = a.hs, GS = a.gv, P = units / hs;
+    auto heads = [&](int u) { return min(GS, a.G - (u / P) * GS); };  // query heads of unit u
     auto eff_len = [&](int u) {
-        const int L = a.lens[u];
+        const int L = a.lens[u % P];
         return unit_ok(L, a.L_cap, a.append) ? L + a.append : -1;
     };
     // stage the lengths in the (still idle) ring memory with one coalesced sweep; the
@@ -319,7 +327,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
             const int u = u0 + k * (int)blockDim.x + tid;
-            Lr[k] = u < units ? __ldcg(a.lens + u) : 0;
+            Lr[k] = u < units ? __ldcg(a.lens + u % P) : 0;
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
@@ -457,14 +465,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // k-step j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
     // and + {2,3} (a2).
     auto load_q = [&](const Item &it, uint32_t (&qa)[D / 16][2]) {
-        const long qrow = (long)(it.u / a.Hkv) * a.Hq + (long)(it.u % a.Hkv) * a.G;
+        const int pu = it.u % P;
+        const long qrow = (long)(pu / a.Hkv) * a.Hq + (long)(pu % a.Hkv) * a.G + (it.u / P) * GS;
+        const int nh = heads(it.u);
         const __nv_bfloat16 *qp = reinterpret_cast<const __nv_bfloat16 *>(a.q) + (qrow + g) * D;
 #pragma unroll
         for (int hh = 0; hh < HALVES; ++hh)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 uint4 wv = make_uint4(0, 0, 0, 0);
-                if (g < a.G) wv = *reinterpret_cast<const uint4 *>(qp + 64 * hh + 16 * c + 8 * e);
+                if (g < nh) wv = *reinterpret_cast<const uint4 *>(qp + 64 * hh + 16 * c + 8 * e);
                 const int j = 4 * hh + 2 * e;
                 qa[j][0] = wv.x;
                 qa[j][1] = wv.y;
@@ -499,7 +509,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         if (lane == 0) {
             const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid * Sm + slot]);
             const uint32_t dst = my_ring + slot * STAGE;
-            const int y = pit.u * a.L_cap + pit.k0 + 16 * pblk;
+            const int y = (pit.u % P) * a.L_cap + pit.k0 + 16 * pblk;
             fence_async_shared();
             mbar_expect_tx(bar, STAGE);
 #pragma unroll
@@ -523,13 +533,14 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     while (cur.nblk >= 0) {
         const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
         const int nsplit = cur.nsplit, item = cur.slot, wf = cur.wf, slot0 = cur.slot0;  // partial slots
-        const long lb = u / a.Hkv;
-        const int h = u % a.Hkv;
-        const int G = a.G;
-        const __nv_bfloat16 *kn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.k_new) + (long)u * D : nullptr;
-        const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)u * D : nullptr;
-        const long qrow0 = lb * a.Hq + (long)h * G;
-        const int row0 = u * a.L_cap;  // first tensor-map row of this unit
+        const int pu = u % P;  // the cache unit
+        const long lb = pu / a.Hkv;
+        const int h = pu % a.Hkv;
+        const int G = heads(u);
+        const __nv_bfloat16 *kn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.k_new) + (long)pu * D : nullptr;
+        const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)pu * D : nullptr;
+        const long qrow0 = lb * a.Hq + (long)h * a.G + (u / P) * GS;
+        const int row0 = pu * a.L_cap;  // first tensor-map row of this unit
 
         // start this item's copies before the wait on its query registers below
         __syncwarp();
@@ -665,7 +676,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         l += __shfl_xor_sync(0xffffffffu, l, 2);
 
         // the warp that covers the appended index writes the new row into the cache
-        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8)) {
+        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8) && u < P) {
             const bool isv = lane >= D / 8;
             const int pc = isv ? lane - D / 8 : lane;
             __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(isv ? a.V : a.K) + ((long)row0 + Lapp) * D + pc * 8;
@@ -693,7 +704,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             }
             if (c == 0 && g < G) put_lse(a, rs, qrow0 + g, l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY);
         } else {
-            float *po = a.part_o + (size_t)item * G * D;
+            float *po = a.part_o + (size_t)item * GS * D;
 #pragma unroll
             for (int hh = 0; hh < HALVES; ++hh) {
                 const int d0 = 64 * hh + 8 * g;
@@ -709,8 +720,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 }
             }
             if (c == 0 && g < G) {
-                a.part_ml[((size_t)item * G + g) * 2 + 0] = m;
-                a.part_ml[((size_t)item * G + g) * 2 + 1] = l;
+                a.part_ml[((size_t)item * GS + g) * 2 + 0] = m;
+                a.part_ml[((size_t)item * GS + g) * 2 + 1] = l;
             }
             // publish: the warp barrier orders every lane's partial writes before lane 0's
             // release; the last arriver's acquire (and the barrier after it) orders its reads
@@ -731,7 +742,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 #pragma unroll
                         for (int qq = 0; qq < 8; ++qq)
                             if (qq < G)
-                                Mq[qq] = fmaxf(Mq[qq], __ldcg(a.part_ml + ((size_t)(s2 ? 2 * (wf + s2) : slot0) * G + qq) * 2));
+                                Mq[qq] = fmaxf(Mq[qq], __ldcg(a.part_ml + ((size_t)(s2 ? 2 * (wf + s2) : slot0) * GS + qq) * 2));
                     }
                 }
 #pragma unroll
@@ -748,7 +759,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                 }
 #pragma unroll 2
                 for (int s2 = 0; s2 < nsplit; ++s2) {
-                    const size_t it0 = (size_t)(s2 ? 2 * (wf + s2) : slot0) * G;
+                    const size_t it0 = (size_t)(s2 ? 2 * (wf + s2) : slot0) * GS;
 #pragma unroll
                     for (int qq = 0; qq < 8; ++qq) {
                         if (qq < G && Mq[qq] != -INFINITY) {
@@ -815,17 +826,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             // 16 independent loads per lane in flight before any store: a few L2 round
             // trips for the whole grid instead of one per 32 units
             constexpr int BATCH = 16;
-            for (int u0 = 0; u0 < units; u0 += 32 * BATCH) {
+            const int cu = units / hs;  // cache units
+            for (int u0 = 0; u0 < cu; u0 += 32 * BATCH) {
                 int L[BATCH];
 #pragma unroll
                 for (int k = 0; k < BATCH; ++k) {
                     const int u = u0 + 32 * k + lane;
-                    L[k] = u < units ? __ldcg(a.lens + u) : -1;
+                    L[k] = u < cu ? __ldcg(a.lens + u) : -1;
                 }
 #pragma unroll
                 for (int k = 0; k < BATCH; ++k) {
                     const int u = u0 + 32 * k + lane;
-                    if (u < units && unit_ok(L[k], a.L_cap, a.append)) a.lens[u] = L[k] + 1;
+                    if (u < cu && unit_ok(L[k], a.L_cap, a.append)) a.lens[u] = L[k] + 1;
                 }
             }
         }
@@ -885,23 +897,32 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
     // partial slots: two per warp of the grid
     const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.part_slots;
-    if (kv.dtype == RECO_BF16 && a.G <= 8 && a.units <= kMaxTmaUnits && rows < (1ull << 31) && slots_fit) {
+    // the TMA path takes up to 8 query heads per unit; a unit of G <= 16 heads is two
+    // virtual units of ceil(G / 2) heads each
+    a.hs = a.G > 8 ? 2 : 1;
+    a.gv = (a.G + a.hs - 1) / a.hs;
+    if (kv.dtype == RECO_BF16 && a.G <= 16 && (long long)a.units * a.hs <= kMaxTmaUnits && rows < (1ull << 31) &&
+        slots_fit) {
+        DecodeArgs at = a;  // virtual units
+        at.units *= at.hs;
         CUtensorMap mk, mv;
         if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {
             // the counters are zero on entry (zero-filled workspace) and every launch leaves them so
             cudaError_t e;
-            const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(a.units) : tma_smem_bytes<128>(a.units);
+            const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(at.units) : tma_smem_bytes<128>(at.units);
             const void *fn = kv.d == 64 ? (const void *)decode_tma<64> : (const void *)decode_tma<128>;
             e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
             const int grid = device_sm_count();
             if (kv.d == 64)
-                e = launch_pdl(decode_tma<64>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, a);
+                e = launch_pdl(decode_tma<64>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, at);
             else
-                e = launch_pdl(decode_tma<128>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, a);
+                e = launch_pdl(decode_tma<128>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, at);
             return e != cudaSuccess ? e : cudaGetLastError();
         }
     }
+    a.hs = 1;
+    a.gv = a.G;
     const unsigned grid = (unsigned)a.units;
     if (kv.dtype == RECO_F32) {
         if (kv.d == 64) decode_simt<float, 64><<<grid, 128, 0, s>>>(a);

@@ -162,3 +162,28 @@ def test_tma_path_unit_limit(shape):
     lens = rng.integers(1, 41, (layers, batch, h_kv)).astype(np.int32)
     assert lens.size in (8192, 8193)
     _check(wl, lens, True)
+
+
+@pytest.mark.parametrize("h_q,h_kv", [(16, 2), (12, 1), (9, 3)])
+def test_bf16_decode_more_than_8_heads_per_kv_head(h_q, h_kv):
+    """G = 8, 12, 3 ... and 16, 12, 9 heads per KV head: the TMA path takes a unit of more than
+    8 heads as two units of ceil(G / 2) heads over the same rows; ragged lengths, appends (the
+    new row written once), three steps, bf16 and fp32 output."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=3, h_q=h_q, h_kv=h_kv, L=2000, decode_steps=3)
+    rng = np.random.default_rng(h_q)
+    hi = wl.L_cap - 3
+    lens = rng.integers(1, hi + 1, (2, 3, h_kv)).astype(np.int32)
+    lens[0, 0, 0] = hi
+    lens[1, 2, -1] = 1
+    _check(wl, lens, True, steps=3)
+    _check(wl, lens, True, torch.bfloat16, steps=1)
+
+
+def test_bf16_decode_g16_long_units_cut_between_warps():
+    """G = 16 with units long enough to be cut over many warps (partial merges of both halves
+    of every unit), in the deep-ring partition."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=4, h_q=32, h_kv=2, L=40000, decode_steps=2)
+    rng = np.random.default_rng(77)
+    lens = rng.integers(30000, 40001, (2, 4, 2)).astype(np.int32)
+    lens[0, 0, 0] = 5
+    _check(wl, lens, True, steps=2)

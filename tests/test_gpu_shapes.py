@@ -25,7 +25,7 @@ CASES = {
     "mha_g1": dict(h_q=4, h_kv=4, w=16, L=900),            # G = 1
     "g3_d64_pool3": dict(h_q=6, h_kv=2, w=8, d=64, pool=3, L=700),
     "g8_r256": dict(h_q=16, h_kv=2, w=32, L=1300),         # tensor decode at G = 8; pass 2 N = 256
-    "g16_simt_decode": dict(h_q=16, h_kv=1, w=16, L=800),  # G = 16: bf16 decode on the SIMT path
+    "g16_split_decode": dict(h_q=16, h_kv=1, w=16, L=800),  # G = 16: the TMA decode as two 8-head units
     "w1_pool1": dict(w=1, pool=1, L=600),                  # one window query, Eq. 2 without pooling
     "r320_pool9": dict(h_q=10, h_kv=2, w=64, pool=9, L=1500),  # 32B-class window: 3 query tiles, 4 x 80 columns
     "r384": dict(h_q=12, h_kv=2, w=64, L=1000),            # 3 query tiles, full
