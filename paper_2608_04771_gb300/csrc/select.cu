@@ -13,10 +13,10 @@
 //
 // compact_rows: one CTA per (unit, K|V, 128-byte column slice).  kept[] is strictly
 // increasing, so kept[r] >= r (the kernel refuses any index that is not): the source
-// of destination r is never a row that an earlier destination overwrote.  Each CTA walks its destinations in order, reads a
-// chunk of source rows, synchronises, then writes the chunk; reads of later chunks
-// may run ahead of earlier writes because their sources lie above every row written
-// so far.  Rows with kept[r] == r are not moved.
+// of destination r is never a row that an earlier destination overwrote.  Each CTA walks
+// its destinations in chunks, in order: a chunk's reads, a barrier, then its writes;
+// the next chunk's reads are issued before the current chunk's writes, since their
+// sources lie above every row written so far.  Rows with kept[r] == r are not moved.
 #include "common.cuh"
 #include "internal.h"
 
@@ -371,7 +371,7 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
                                                     Count cnt, int L_cap, int row_bytes, unsigned *err)
 {
     constexpr int P = 8;  // 16-byte pieces per 128-byte slice
-    constexpr int U = 2;  // rows per thread in flight
+    constexpr int U = 2;  // rows per thread in one chunk
     const long u = blockIdx.x;
     int lim;
     const int m = cnt.rows(u, err, lim);
@@ -381,9 +381,8 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
     const int rows_per_pass = blockDim.x / P;
     const int my_row = threadIdx.x / P;
     const int off = blockIdx.z * 128 + (threadIdx.x % P) * 16;
-    for (int r0 = 0; r0 < m; r0 += U * rows_per_pass) {
-        uint4 v[U];
-        int dst[U];
+    const int step = U * rows_per_pass;  // destinations per chunk
+    auto load = [&](int r0, uint4 (&v)[U], int (&dst)[U]) {
 #pragma unroll
         for (int i = 0; i < U; ++i) {
             const int r = r0 + i * rows_per_pass + my_row;
@@ -398,10 +397,26 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
                 }
             }
         }
-        __syncthreads();
+    };
+    auto store = [&](const uint4 (&v)[U], const int (&dst)[U]) {
 #pragma unroll
         for (int i = 0; i < U; ++i)
             if (dst[i] >= 0) *reinterpret_cast<uint4 *>(base + (long)dst[i] * row_bytes + off) = v[i];
+    };
+    // Two chunks in registers: the next chunk's reads are issued before this chunk's
+    // writes (its sources lie at or above its first destination, above every row this
+    // chunk writes); the barrier before a chunk's writes follows every read of it.
+    uint4 va[U], vb[U];
+    int da[U], db[U];
+    load(0, va, da);
+    for (int r0 = 0; r0 < m; r0 += 2 * step) {
+        load(r0 + step, vb, db);
+        __syncthreads();
+        store(va, da);
+        if (r0 + step >= m) break;
+        load(r0 + 2 * step, va, da);
+        __syncthreads();
+        store(vb, db);
     }
 }
 
