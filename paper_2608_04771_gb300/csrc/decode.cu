@@ -270,7 +270,7 @@ size_t tma_smem_bytes(int units)
 // Byte offset of 16-byte chunk ch (0..7) of row rr inside a 128B-swizzled 16-row box.
 __device__ __forceinline__ uint32_t swz(int rr, int ch) { return rr * 128 + ((ch ^ (rr & 7)) << 4); }
 
-template <int D>
+template <int D, int HS>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     decode_tma(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, DecodeArgs a)
 {
@@ -313,10 +313,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // unit u % P (P cache units).  With two halves (G > 8) all first halves come first in
     // the plan, then all second halves in the same order, so warps w and w + W/2 stream
     // the same rows at about the same time and the second read mostly hits L2.
-    const int hs = a.hs, GS = a.gv, P = units / hs;
-    auto heads = [&](int u) { return min(GS, a.G - (u / P) * GS); };  // query heads of unit u
+    const int GS = a.gv, P = units / HS;
+    auto cache_unit = [&](int u) { return HS == 1 ? u : u % P; };
+    auto head_part = [&](int u) { return HS == 1 ? 0 : u / P; };
     auto eff_len = [&](int u) {
-        const int L = a.lens[u % P];
+        const int L = a.lens[cache_unit(u)];
         return unit_ok(L, a.L_cap, a.append) ? L + a.append : -1;
     };
     // stage the lengths in the (still idle) ring memory with one coalesced sweep; the
@@ -327,7 +328,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
             const int u = u0 + k * (int)blockDim.x + tid;
-            Lr[k] = u < units ? __ldcg(a.lens + u % P) : 0;
+            Lr[k] = u < units ? __ldcg(a.lens + cache_unit(u)) : 0;
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
@@ -388,7 +389,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // (its last piece): only those two pieces of a warp can be partial.  Only long units
     // are cut, and no range start moves inside a long unit, so there the ideal owners hold.
     struct Item {
-        int u, ub, wf, nsplit, slot, slot0, le, k0, k1, Lapp, nblk;
+        int u, pu, hp, ub, wf, nsplit, slot, slot0, le, k0, k1, Lapp, nblk;  // pu, hp: cache unit, head part
     };
     auto last_le = [](const int *pre, int units_, int d) {  // largest u with pre[u] <= d
         int lo = 0, hi = units_ - 1;
@@ -421,6 +422,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             const int bend = min(b_end, ue);
             const int le_raw = eff_len(u);
             it.u = u;
+            it.pu = cache_unit(u);
+            it.hp = head_part(u);
             it.ub = ub;
             it.le = le_raw >= 0 ? le_raw : 0;
             it.Lapp = (le_raw >= 0 && a.append) ? it.le - 1 : -1;
@@ -446,6 +449,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             if (pb[u + 1] == pb[u]) {
                 const int le_raw = eff_len(u);
                 it.u = u;
+                it.pu = cache_unit(u);
+                it.hp = head_part(u);
                 it.ub = pb[u];
                 it.le = 0;
                 it.Lapp = -1;
@@ -465,9 +470,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // k-step j = 4*hh + 2*e + half takes elements 64*hh + 16c + 8e + 4*half + {0,1} (a0)
     // and + {2,3} (a2).
     auto load_q = [&](const Item &it, uint32_t (&qa)[D / 16][2]) {
-        const int pu = it.u % P;
-        const long qrow = (long)(pu / a.Hkv) * a.Hq + (long)(pu % a.Hkv) * a.G + (it.u / P) * GS;
-        const int nh = heads(it.u);
+        const long qrow = (long)(it.pu / a.Hkv) * a.Hq + (long)(it.pu % a.Hkv) * a.G + it.hp * GS;
+        const int nh = min(GS, a.G - it.hp * GS);
         const __nv_bfloat16 *qp = reinterpret_cast<const __nv_bfloat16 *>(a.q) + (qrow + g) * D;
 #pragma unroll
         for (int hh = 0; hh < HALVES; ++hh)
@@ -509,7 +513,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         if (lane == 0) {
             const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&bars[wid * Sm + slot]);
             const uint32_t dst = my_ring + slot * STAGE;
-            const int y = (pit.u % P) * a.L_cap + pit.k0 + 16 * pblk;
+            const int y = pit.pu * a.L_cap + pit.k0 + 16 * pblk;
             fence_async_shared();
             mbar_expect_tx(bar, STAGE);
 #pragma unroll
@@ -533,13 +537,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     while (cur.nblk >= 0) {
         const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
         const int nsplit = cur.nsplit, item = cur.slot, wf = cur.wf, slot0 = cur.slot0;  // partial slots
-        const int pu = u % P;  // the cache unit
+        const int pu = cur.pu;  // the cache unit
         const long lb = pu / a.Hkv;
         const int h = pu % a.Hkv;
-        const int G = heads(u);
+        const int G = min(GS, a.G - cur.hp * GS);
         const __nv_bfloat16 *kn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.k_new) + (long)pu * D : nullptr;
         const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)pu * D : nullptr;
-        const long qrow0 = lb * a.Hq + (long)h * a.G + (u / P) * GS;
+        const long qrow0 = lb * a.Hq + (long)h * a.G + cur.hp * GS;
         const int row0 = pu * a.L_cap;  // first tensor-map row of this unit
 
         // start this item's copies before the wait on its query registers below
@@ -676,7 +680,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         l += __shfl_xor_sync(0xffffffffu, l, 2);
 
         // the warp that covers the appended index writes the new row into the cache
-        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8) && u < P) {
+        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8) && cur.hp == 0) {
             const bool isv = lane >= D / 8;
             const int pc = isv ? lane - D / 8 : lane;
             __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(isv ? a.V : a.K) + ((long)row0 + Lapp) * D + pc * 8;
@@ -826,7 +830,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             // 16 independent loads per lane in flight before any store: a few L2 round
             // trips for the whole grid instead of one per 32 units
             constexpr int BATCH = 16;
-            const int cu = units / hs;  // cache units
+            const int cu = units / HS;  // cache units
             for (int u0 = 0; u0 < cu; u0 += 32 * BATCH) {
                 int L[BATCH];
 #pragma unroll
@@ -910,14 +914,19 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
             // the counters are zero on entry (zero-filled workspace) and every launch leaves them so
             cudaError_t e;
             const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(at.units) : tma_smem_bytes<128>(at.units);
-            const void *fn = kv.d == 64 ? (const void *)decode_tma<64> : (const void *)decode_tma<128>;
+            const bool two = at.hs == 2;
+            const void *fn = kv.d == 64 ? (two ? (const void *)decode_tma<64, 2> : (const void *)decode_tma<64, 1>)
+                                        : (two ? (const void *)decode_tma<128, 2> : (const void *)decode_tma<128, 1>);
             e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
             const int grid = device_sm_count();
+            const dim3 blk(kDecodeWarps * 32);
             if (kv.d == 64)
-                e = launch_pdl(decode_tma<64>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, at);
+                e = two ? launch_pdl(decode_tma<64, 2>, dim3(grid), blk, smem, s, mk, mv, at)
+                        : launch_pdl(decode_tma<64, 1>, dim3(grid), blk, smem, s, mk, mv, at);
             else
-                e = launch_pdl(decode_tma<128>, dim3(grid), dim3(kDecodeWarps * 32), smem, s, mk, mv, at);
+                e = two ? launch_pdl(decode_tma<128, 2>, dim3(grid), blk, smem, s, mk, mv, at)
+                        : launch_pdl(decode_tma<128, 1>, dim3(grid), blk, smem, s, mk, mv, at);
             return e != cudaSuccess ? e : cudaGetLastError();
         }
     }
