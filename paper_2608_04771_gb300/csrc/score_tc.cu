@@ -125,7 +125,9 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
 }
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row atoms of
-// 1024 bytes (stride byte offset 1024), descriptor version 1.
+// 1024 bytes (stride byte offset 1024), descriptor version 1.  The start address sits in
+// the low 14 bits as address / 16; a shared-memory address stays below 2^18 bytes, so
+// the descriptor of (address + offset) is this one plus offset / 16 (no carry out).
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
 {
     uint64_t d = 0;
@@ -381,12 +383,14 @@ __global__ void __launch_bounds__(Pass1Cfg<D, MT, N, EG>::THREADS, 1)
                         }
                         tc_fence_after();
                         const uint32_t d = tmem + (uint32_t)(b * N);
+                        // descriptors of the first K slice; later slices add their offset / 16
+                        const uint64_t ad0 = sw128_desc(Qs + mt * HALVES * QBOX);
+                        const uint64_t bd0 = sw128_desc(Ks + s * KSTAGE);
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k) {
                             const int hh = k >> 2, kk = k & 3;
-                            const uint64_t ad = sw128_desc(Qs + (mt * HALVES + hh) * QBOX + kk * 32);
-                            const uint64_t bd = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
-                            tc_mma(d, ad, bd, IDESC, k > 0 ? 1u : 0u);
+                            tc_mma(d, ad0 + (uint64_t)((hh * QBOX + kk * 32) >> 4),
+                                   bd0 + (uint64_t)((hh * KBOX + kk * 32) >> 4), IDESC, k > 0 ? 1u : 0u);
                         }
                         tc_commit(smem_addr(&bar_afull[b]));
                     }
@@ -630,12 +634,15 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                         }
                         tc_fence_after();
                         const uint32_t d = tmem + (uint32_t)(b * stride);
+                        // descriptors of the first K slice; later slices add their offset / 16
+                        const uint64_t ad0 = sw128_desc(Ks + s * KSTAGE);
+                        const uint64_t bd0 = sw128_desc(Qs + h * NW * 128);
+                        const uint64_t bh16 = (uint64_t)(QBOXB >> 4);
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k) {
                             const int hh = k >> 2, kk = k & 3;
-                            const uint64_t ad = sw128_desc(Ks + s * KSTAGE + hh * KBOX + kk * 32);
-                            const uint64_t bd = sw128_desc(Qs + hh * QBOXB + h * NW * 128 + kk * 32);
-                            tc_mma(d, ad, bd, idesc, k > 0 ? 1u : 0u);
+                            tc_mma(d, ad0 + (uint64_t)((hh * KBOX + kk * 32) >> 4), bd0 + hh * bh16 + (uint64_t)(kk * 2),
+                                   idesc, k > 0 ? 1u : 0u);
                         }
                         tc_commit(smem_addr(&bar_afull[b]));
                     }
