@@ -161,3 +161,53 @@ def test_penalty_sample_validates_before_launch(L):
     assert call(V=4096 * 1024 + 1) == reco.RECO_EUNSUPPORTED
     assert call(beta=-1.0) == reco.RECO_EINVAL
     assert call(B=0) == reco.RECO_EINVAL
+
+
+def test_split_select_compact_and_ring_decode_validate_before_launch(L):
+    """reco_select_topm, reco_compact and reco_decode_attn_ring reject bad arguments on the
+    host, before any launch."""
+    kv = _kv()
+    vp = ctypes.c_void_p
+    ws = vp(256 * 1000)
+    big = 1 << 30
+    st = L.reco_select_topm(ctypes.byref(kv), vp(16), vp(16), vp(16), 16, None, ws, big, None)
+    assert st == reco.RECO_EINVAL and b"kept_idx" in L.reco_last_error()
+    st = L.reco_select_topm(ctypes.byref(kv), vp(16), vp(16), vp(16), 0, vp(16), ws, big, None)
+    assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
+    st = L.reco_select_topm(ctypes.byref(kv), vp(16), vp(16), vp(18), 16, vp(16), ws, big, None)
+    assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    st = L.reco_select_topm(ctypes.byref(kv), vp(16), vp(16), vp(16), 16, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    # the selection alone does not touch the cache: NULL K/V pointers are accepted there ...
+    st = L.reco_select_topm(ctypes.byref(_kv(k=0, v=0)), vp(16), vp(16), vp(16), 16, vp(16), ws, 10, None)
+    assert st == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    # ... but not by the compaction
+    st = L.reco_compact(ctypes.byref(_kv(k=0, v=0)), vp(16), vp(16), vp(16), 16, None)
+    assert st == reco.RECO_EINVAL and b"NULL" in L.reco_last_error()
+    st = L.reco_compact(ctypes.byref(kv), vp(16), vp(16), None, 16, None)
+    assert st == reco.RECO_EINVAL and b"keep" in L.reco_last_error()
+    st = L.reco_compact(ctypes.byref(kv), vp(17), vp(16), vp(16), 16, None)
+    assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    st = L.reco_compact(ctypes.byref(kv), vp(16), vp(16), vp(16), 101, None)
+    assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
+    dec = lambda kv_, ring, slots, slot: L.reco_decode_attn_ring(  # noqa: E731
+        ctypes.byref(kv_), vp(16), None, None, vp(16), 0.1, vp(16), 0, ring, slots, slot, ws, 10, None)
+    assert dec(kv, vp(16), 0, vp(16)) == reco.RECO_EINVAL and b"slots" in L.reco_last_error()
+    assert dec(kv, None, 4, vp(16)) == reco.RECO_EINVAL
+    assert dec(kv, vp(16), 4, vp(20)) == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    # past its own checks it applies reco_decode_attn's (here: the workspace is too short)
+    assert dec(kv, vp(16), 4, vp(16)) == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
+    assert dec(_kv(H_q=34, H_kv=2), vp(16), 4, vp(16)) == reco.RECO_EUNSUPPORTED
+
+
+def test_decode_workspace_counts_a_ticket_per_half_unit_above_8_heads(L):
+    """A unit of more than 8 query heads per KV head runs as two units on the tensor path, with
+    a merge ticket each: the workspace holds one more int per unit."""
+    w8 = reco.reco_workspace_bytes(reco.RECO_OP_DECODE, _kv(H_q=16, H_kv=2))
+    w16 = reco.reco_workspace_bytes(reco.RECO_OP_DECODE, _kv(H_q=32, H_kv=2))
+    parts = 4096  # partial slots, each G x (2 + d) floats
+    assert w16 - w8 >= parts * 8 * (2 + 128) * 4  # the partials of 8 more heads per slot
+    kv = _kv(H_q=32, H_kv=2, n_layers=64, B=16)  # 2048 units: the counters alone differ by 8 KB
+    kv8 = _kv(H_q=16, H_kv=2, n_layers=64, B=16)
+    g = reco.reco_workspace_bytes(reco.RECO_OP_DECODE, kv) - reco.reco_workspace_bytes(reco.RECO_OP_DECODE, kv8)
+    assert g >= parts * 8 * (2 + 128) * 4 + 2048 * 4 - 512
