@@ -723,10 +723,10 @@ def run_trace(args):
     if args.generated:
         spec.generated = args.generated
     use_graph = not args.no_graph
-    warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64, use_graph=use_graph)
+    warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=32, use_graph=use_graph)
     warm.run(max_tokens=128)
     torch.cuda.synchronize()
-    tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=64, use_graph=use_graph)
+    tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=32, use_graph=use_graph)
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.perf_counter()
@@ -748,12 +748,14 @@ def run_trace(args):
         "config": {"workload": f"trace: 7B-class heads, 28 layers, batch {spec.batch}, prompt {spec.prompt}, "
                                f"{spec.generated} generated tokens, steps Poisson({spec.step_mean})+{spec.step_min}, "
                                f"Beta(2,2) rewards, reading {spec.reading}, interval S={spec.interval}",
-                   "inputs": "per-token synthetic inputs drawn once for 64 tokens and reused cyclically",
-                   "window": "Eq. 2's window queries are the last w decoded tokens' queries; a boundary scores "
-                             "in one pass with their decode lse (kept in a device ring) when none of the "
-                             "compressing sequences was compressed within the window, else in two passes",
-                   "per_token_launch": "captured CUDA graph (input gather from the pool + decode writing its lse "
-                                       "into the ring + penalty and draw)" if use_graph else "direct calls"},
+                   "inputs": "per-token synthetic inputs drawn once for w = 32 tokens and reused cyclically",
+                   "window": "Eq. 2's window queries are the last w decoded tokens' queries; their queries and "
+                             "decode lse are kept in device rings of w slots by every token, and a boundary "
+                             "scores in one pass with those lse when none of the compressing sequences was "
+                             "compressed within the window, else in two passes",
+                   "per_token_launch": "captured CUDA graph (input gather from the pool + query into the window "
+                                       "ring + decode writing its lse into the ring + penalty and draw in one "
+                                       "launch)" if use_graph else "direct calls"},
         "trace": {"generated": ev.generated, "decode_launches": ev.tokens, "steps_completed": ev.steps_completed,
                   "compressions": ev.compressions, "probes": len(ev.probes),
                   "boundary_scorings": {"one_pass_decode_lse": ev.lse_scorings, "two_pass": ev.two_pass_scorings},

@@ -146,6 +146,9 @@ reco_status reco_score_cache(const reco_kv *kv, const void *q_win, const int32_t
  *            vouches for that correspondence: no compression of the unit between
  *            those decodes and this call.  A non-finite entry sets the device
  *            error word; that row then adds nothing to the scores.
+ * Every candidate key (j < L-w) precedes the whole window, so each row's term of
+ * Eq. 2 needs only its query and its normaliser: the window rows may come in any
+ * order, as long as q_win row t and row_lse row t belong to the same token.
  * Every other argument, the result and the workspace are those of
  * reco_score_cache.                                                             */
 reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int32_t *lens, const int32_t *keep,
@@ -243,13 +246,20 @@ reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new
  * *slot to (*slot + 1) % slots, all on the device, so a captured graph decodes every
  * token with no separate push.  It is reco_decode_attn followed by reco_lse_push in one
  * launch, with the same results.
- *   ring : [2 * slots][n_layers * B * H_q] float32 (device, two rows written)
- *   slot : int64 (device, read and advanced); a value outside [0, slots) writes no ring
- *          row, leaves *slot as it is and sets the device error word
+ *   ring   : [2 * slots][n_layers * B * H_q] float32 (device, two rows written)
+ *   slot   : int64 (device, read and advanced); a value outside [0, slots) writes no
+ *            ring row, leaves *slot as it is and sets the device error word
+ *   q_ring : [n_layers][B][H_q][slots][d], the cache dtype, 16-byte aligned (device),
+ *            or NULL: row *slot of every query head's `slots` rows receives that
+ *            head's query.  With slots = w it then holds the queries of the last w
+ *            tokens in slot order (token t in slot t mod w), the same order as ring
+ *            rows 0..w-1: together the q_win and row_lse of reco_score_cache_lse, with
+ *            no gather (its result does not depend on the order of the window rows).
  * Every other argument, the result and the workspace are those of reco_decode_attn.    */
 reco_status reco_decode_attn_ring(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,
                                   int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *ring,
-                                  int slots, int64_t *slot, void *ws, size_t ws_bytes, cudaStream_t stream);
+                                  int slots, int64_t *slot, void *q_ring, void *ws, size_t ws_bytes,
+                                  cudaStream_t stream);
 
 /* Eq. 3 + Eq. 4 (Sec. 3.3, reward-banded reflection penalty), in place:
  *   beta_b = 0, beta/2 or beta by the band of rewards[b] (float32 compares);
@@ -276,7 +286,9 @@ reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids
  *            (the logits are penalised in place exactly as reco_reflect_penalty does)
  *   uniforms : [B] float32 (device), one draw in [0, 1) per sequence
  *   tokens   : [B] int32 (device, written)
- *   ws       : at least B * reco_workspace_bytes(RECO_OP_SAMPLE, NULL, V) bytes
+ *   ws       : at least B * reco_workspace_bytes(RECO_OP_SAMPLE, NULL, V) bytes (not
+ *              touched when logits are 16-byte aligned, V is a multiple of 4 and
+ *              V <= 393216: then one launch with a cluster of CTAs per row does all)
  * V may be at most 4194304.  The probabilities are float32 (2^x on the special-
  * function unit), so a draw within about 1e-5 of a boundary of the cumulative
  * distribution may select the neighbouring token.                              */

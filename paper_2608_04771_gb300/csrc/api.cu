@@ -346,7 +346,8 @@ reco_status reco_compact(const reco_kv *kv, const int32_t *kept_idx, int32_t *le
 namespace {
 reco_status decode_checked(const reco_kv *kv, const void *q, const void *k_new, const void *v_new, int32_t *lens,
                            float scale, void *out, reco_dtype out_dtype, float *lse, float *ring, int slots,
-                           int64_t *slot, void *ws, size_t ws_bytes, cudaStream_t stream, const char *name)
+                           int64_t *slot, void *q_ring, void *ws, size_t ws_bytes, cudaStream_t stream,
+                           const char *name)
 {
     reco_status st = check_kv(kv);
     if (st != RECO_OK) return st;
@@ -364,7 +365,7 @@ reco_status decode_checked(const reco_kv *kv, const void *q, const void *k_new, 
     unsigned *err;
     if ((st = error_word(&err)) != RECO_OK) return st;
     cudaError_t e = reco::launch_decode(*kv, q, k_new, v_new, lens, scale, out, out_dtype, lse, lay, err, stream, ring,
-                                        slots, reinterpret_cast<long long *>(slot));
+                                        slots, reinterpret_cast<long long *>(slot), q_ring);
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, name);
 }
 }  // namespace
@@ -375,19 +376,20 @@ reco_status reco_decode_attn(const reco_kv *kv, const void *q, const void *k_new
                              float scale, void *out, reco_dtype out_dtype, float *lse, void *ws, size_t ws_bytes,
                              cudaStream_t stream)
 {
-    return decode_checked(kv, q, k_new, v_new, lens, scale, out, out_dtype, lse, nullptr, 0, nullptr, ws, ws_bytes,
-                          stream, "reco_decode_attn launch");
+    return decode_checked(kv, q, k_new, v_new, lens, scale, out, out_dtype, lse, nullptr, 0, nullptr, nullptr, ws,
+                          ws_bytes, stream, "reco_decode_attn launch");
 }
 
 reco_status reco_decode_attn_ring(const reco_kv *kv, const void *q, const void *k_new, const void *v_new,
                                   int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *ring, int slots,
-                                  int64_t *slot, void *ws, size_t ws_bytes, cudaStream_t stream)
+                                  int64_t *slot, void *q_ring, void *ws, size_t ws_bytes, cudaStream_t stream)
 {
     if (slots < 1 || !ring || !slot) return fail(RECO_EINVAL, "need slots >= 1 and non-NULL ring and slot");
     if (((uintptr_t)ring & 3u) || ((uintptr_t)slot & 7u))
         return fail(RECO_EINVAL, "ring must be 4-byte aligned, slot 8-byte aligned");
-    return decode_checked(kv, q, k_new, v_new, lens, scale, out, out_dtype, nullptr, ring, slots, slot, ws, ws_bytes,
-                          stream, "reco_decode_attn_ring launch");
+    if (q_ring && !al16(q_ring)) return fail(RECO_EINVAL, "q_ring must be 16-byte aligned");
+    return decode_checked(kv, q, k_new, v_new, lens, scale, out, out_dtype, nullptr, ring, slots, slot, q_ring, ws,
+                          ws_bytes, stream, "reco_decode_attn_ring launch");
 }
 
 reco_status reco_reflect_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,

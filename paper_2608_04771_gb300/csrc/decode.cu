@@ -5,6 +5,8 @@
 // SM (for long work 4 of them, each with a ring twice as deep).  Every CTA first builds the same work plan from lens: the prefix sum of 16-key
 // blocks per unit, with the blocks of all units laid end to end and cut into one equal
 // contiguous range per warp (a stream-K split: balanced to one block, no work queue).
+// When no unit is long enough to be cut, the units are instead sorted by length and
+// dealt whole to the warps in snake order (longest first).
 // An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
 // (128-byte swizzled 16 x 64 tiles of K and V) into the warp's 3-stage ring and the
 // warp waits on the stage's mbarrier (bounded).  QK^T and PV run on mma.sync
@@ -20,6 +22,8 @@
 //
 // float32 path (decode_simt): one CTA per unit, four warps over the keys, G <= 16.
 #include <cuda.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "internal.h"
@@ -68,6 +72,8 @@ struct DecodeArgs {
     long long *slot;  // device ring row, advanced by one (mod slots) per launch
     int slots;
     long long nq;     // query heads of the launch (layers * B * H_q)
+    void *qring;      // or nullptr: [nq][slots][D] of q's dtype, row *slot of every head gets its query
+    int q_bytes;      // bytes per element of q
 };
 
 // The ring row this launch writes (read once the previous kernel's writes are visible),
@@ -98,6 +104,13 @@ __device__ __forceinline__ int atom_add_acq_rel(int *p, int v)
 {
     int old;
     asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+__device__ __forceinline__ unsigned long long atom_add_acq_rel_u64(unsigned long long *p, unsigned long long v)
+{
+    unsigned long long old;
+    asm volatile("atom.acq_rel.gpu.global.add.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
     return old;
 }
 
@@ -259,7 +272,8 @@ template <int D> struct TmaLayout {
 
 // the largest plan fits beside the d = 128 ring (227 KB per CTA, about 1 KB of it static)
 static_assert(1024 + TmaLayout<128>::RING + (kMaxTmaUnits + 1) * 4 + 1024 <= 227 * 1024, "decode smem budget");
-static_assert(kMaxTmaUnits * 4 <= TmaLayout<64>::RING, "lengths are staged in the ring");
+static_assert((kMaxTmaUnits + 32 + (kMaxWholeBlocks + 1) * kDecodeWarps * 32) * 4 <= TmaLayout<64>::RING,
+              "lengths and the sort counters are staged in the ring");
 
 template <int D>
 size_t tma_smem_bytes(int units)
@@ -281,6 +295,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NW * S];  // ring stages of all warps (either partition)
     __shared__ int sm_scan[NW];
+    __shared__ int sm_red[2 * NW];  // per warp: most blocks of a unit, units with keys
     const uint32_t raw0 = (uint32_t)__cvta_generic_to_shared(smem_raw);
     const uint32_t ring0 = (raw0 + 1023u) & ~1023u;
     int *sm_pre = reinterpret_cast<int *>(smem_raw + (ring0 - raw0) + LY::RING);  // [units + 1]
@@ -343,15 +358,26 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
     __syncthreads();
     {
-        int my_b = 0;
-        for (int u = u_lo; u < u_hi; ++u) my_b += (len_sm[u] + 15) >> 4;
+        int my_b = 0, my_max = 0, my_ne = 0;
+        for (int u = u_lo; u < u_hi; ++u) {
+            const int nb = (len_sm[u] + 15) >> 4;
+            my_b += nb;
+            my_max = max(my_max, nb);
+            my_ne += nb > 0;
+        }
         int f = my_b;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int nf = __shfl_up_sync(0xffffffffu, f, o);
             if (lane >= o) f += nf;
         }
+        my_max = __reduce_max_sync(0xffffffffu, (unsigned)my_max);
+        my_ne = __reduce_add_sync(0xffffffffu, (unsigned)my_ne);
         if (lane == 31) sm_scan[wid] = f;
+        if (lane == 0) {
+            sm_red[wid] = my_max;
+            sm_red[NW + wid] = my_ne;
+        }
         __syncthreads();
         int rb = f - my_b;
         for (int w2 = 0; w2 < wid; ++w2) rb += sm_scan[w2];
@@ -373,6 +399,52 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // pieces, whose merges cost more than the shallower rings save.
     const bool deep =
         NB >= kDeepBlocksPerWarp * total_warps || (NB >= 8 * total_warps && total_warps > 2 * units);
+    int max_nb = 0, n_ne = 0;  // most blocks of one unit; units with keys
+#pragma unroll
+    for (int w2 = 0; w2 < NW; ++w2) {
+        max_nb = max(max_nb, sm_red[w2]);
+        n_ne += sm_red[NW + w2];
+    }
+    // Only short units (none is ever cut): the contiguous deal below would leave some warps
+    // two whole units where others have one.  Instead the units are sorted by blocks, most
+    // first (ties by index, so every CTA builds the same order), and dealt in snake order:
+    // warp w takes sorted units w, 2W-1-w, 2W+w, ... of W = min(warps, units with keys),
+    // so a warp holding one of the longest units in a round holds one of the shortest in
+    // the next.  The order replaces the block prefix in shared memory; units without keys
+    // sort last.
+    const bool snake = !deep && max_nb <= kMaxWholeBlocks;
+    int *order = sm_pre;
+    if (snake) {
+        constexpr int NBK = kMaxWholeBlocks + 1;  // buckets: 16 - blocks, so most blocks first
+        int *cnt = len_sm + ((units + 31) & ~31);  // [NBK][blockDim.x], also in the idle ring
+        for (int k = 0; k < NBK; ++k) cnt[k * blockDim.x + tid] = 0;
+        for (int u = u_lo; u < u_hi; ++u) ++cnt[(kMaxWholeBlocks - ((len_sm[u] + 15) >> 4)) * blockDim.x + tid];
+        __syncthreads();
+        // exclusive scan of cnt in memory order (bucket-major, then thread): thread t takes
+        // entries [NBK t, NBK (t + 1))
+        int loc = 0;
+        for (int k = 0; k < NBK; ++k) loc += cnt[tid * NBK + k];
+        int f = loc;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int nf = __shfl_up_sync(0xffffffffu, f, o);
+            if (lane >= o) f += nf;
+        }
+        __syncthreads();  // every thread has read its entries (and NB, before the order overwrites pb)
+        if (lane == 31) sm_scan[wid] = f;
+        __syncthreads();
+        int run = f - loc;
+        for (int w2 = 0; w2 < wid; ++w2) run += sm_scan[w2];
+        for (int k = 0; k < NBK; ++k) {
+            const int c2 = cnt[tid * NBK + k];
+            cnt[tid * NBK + k] = run;
+            run += c2;
+        }
+        __syncthreads();
+        // each thread places its own units, in index order, from its own column of cnt
+        for (int u = u_lo; u < u_hi; ++u) order[cnt[(kMaxWholeBlocks - ((len_sm[u] + 15) >> 4)) * blockDim.x + tid]++] = u;
+        __syncthreads();
+    }
     bool aborted = false;
     {
     const int NWm = deep ? NW / 2 : NW, Sm = deep ? 2 * S : S;  // NWm * Sm == NW * S either way
@@ -409,13 +481,53 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // static deal interleaved across CTAs (warp wid of every CTA before warp wid+1 of
     // any): with fewer working warps than warps the work still spreads over all SMs
     const int gw = wid * (int)gridDim.x + (int)blockIdx.x;
-    const bool working = gw < W;
+    const bool working = gw < W && !snake;
     const int b_end = working ? snap(wstart(gw + 1)) : 0;
     int b_next = working ? snap(wstart(gw)) : 0;
     int eu = gw;  // next unit this warp checks for emptiness (empty units: no blocks)
+    const int Ws = min(NW * (int)gridDim.x, n_ne);  // snake deal: warps with units
+    int sk = 0, spos = gw < Ws ? gw : n_ne;          // round and sorted position of the next unit
     auto next_item = [&]() {
         Item it;
         it.nblk = -1;  // no item
+        if (snake) {
+            if (spos < n_ne) {
+                const int u = order[spos];
+                const int le_raw = eff_len(u);
+                it.u = u;
+                it.pu = cache_unit(u);
+                it.hp = head_part(u);
+                it.ub = 0;
+                it.le = le_raw >= 0 ? le_raw : 0;
+                it.Lapp = (le_raw >= 0 && a.append) ? it.le - 1 : -1;
+                it.k0 = 0;
+                it.k1 = it.le;
+                it.nblk = (it.le + 15) >> 4;
+                it.wf = gw;
+                it.nsplit = 1;
+                it.slot = it.slot0 = 0;
+                ++sk;
+                spos = sk * Ws + ((sk & 1) ? Ws - 1 - gw : gw);
+                return it;
+            }
+            while (n_ne + eu < units) {  // units without keys: zero output, lse = -inf
+                const int u = order[n_ne + eu];
+                eu += total_warps;
+                it.u = u;
+                it.pu = cache_unit(u);
+                it.hp = head_part(u);
+                it.ub = 0;
+                it.le = 0;
+                it.Lapp = -1;
+                it.k0 = it.k1 = 0;
+                it.nblk = 0;
+                it.wf = 0;
+                it.nsplit = 1;
+                it.slot = it.slot0 = 0;
+                return it;
+            }
+            return it;
+        }
         if (b_next < b_end) {
             const int u = last_le(pb, units, b_next);  // the nonempty unit holding block b_next
             const int ub = pb[u], ue = pb[u + 1];
@@ -533,6 +645,31 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     uint32_t qa_n[D / 16][2];  // query fragments of the next item to start
     if (cur.nblk >= 0) load_q(cur, qa_n);
     nxt = cur.nblk >= 0 ? next_item() : cur;
+    // the launch's queries into the window ring (row rs of every query head's `slots`
+    // rows): each warp copies an equal share of 16-byte chunks while its first copies
+    // are in flight
+    if (a.qring != nullptr && rs >= 0) {
+        constexpr int CH = D / 8;  // 16-byte chunks of a bf16 query row
+        const long long n16 = a.nq * CH;
+        const int tw = (int)gridDim.x * NW, me = (int)blockIdx.x * NW + wid;
+        const long long per = (n16 + tw - 1) / tw;
+        const long long c0 = min(n16, (long long)me * per), c1 = min(n16, c0 + per);
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.q);
+        uint4 *dst = reinterpret_cast<uint4 *>(a.qring);
+        for (long long cb = c0; cb < c1; cb += 32 * 8) {
+            uint4 v[8];  // all loads in flight before the stores
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const long long c = cb + 32 * k + lane;
+                if (c < c1) v[k] = __ldcg(src + c);
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const long long c = cb + 32 * k + lane;
+                if (c < c1) dst[(c / CH * a.slots + rs) * CH + c % CH] = v[k];
+            }
+        }
+    }
 
     while (cur.nblk >= 0) {
         const int u = cur.u, k0 = cur.k0, k1 = cur.k1, Lapp = cur.Lapp;
@@ -810,28 +947,53 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
     }
 
-    // Every warp, stopped early or not, counts itself done (a stopped one marks that
-    // first).  The last one has every other warp behind it: it advances the lengths
-    // (every plan has been read by then) and clears the counters, so a launch leaves the
-    // workspace's counters zero as it found them, also after a stop.
-    int done = 0;
+    // Every warp, stopped early or not, counts itself done with one 64-bit add on the
+    // pair counters[0..1]: +1 on counters[1] (warps done) and, for a stopped warp, +1 on
+    // counters[0] (warps stopped), so the value the add returns tells the last warp of
+    // every stop before it, with no further read.  The last one has every other warp
+    // behind it: it advances the lengths (every plan has been read by then) and clears
+    // the counters, so a launch leaves the workspace's counters zero as it found them,
+    // also after a stop.
+    unsigned long long dc = 0;
+    const bool stopped = __shfl_sync(0xffffffffu, aborted, 0);
     __syncwarp();
-    if (lane == 0) {
-        if (aborted) atomicOr(&a.counters[0], 1);
-        done = atom_add_acq_rel(&a.counters[1], 1);
-    }
-    done = __shfl_sync(0xffffffffu, done, 0);
+    if (lane == 0)
+        dc = atom_add_acq_rel_u64(reinterpret_cast<unsigned long long *>(a.counters),
+                                  (1ull << 32) | (stopped ? 1ull : 0ull));
+    dc = __shfl_sync(0xffffffffu, dc, 0);
     __syncwarp();
-    if (done == total_warps - 1) {
-        const bool any_stop = __ldcg(&a.counters[0]) != 0;
+    if ((int)(dc >> 32) == total_warps - 1) {
+        const bool any_stop = stopped || (uint32_t)dc != 0u;
         if (any_stop) {  // tickets of units whose pieces stopped early may still count
             for (int u = lane; u < units; u += 32) a.counters[2 + u] = 0;
         } else if (a.append) {
-            // 16 independent loads per lane in flight before any store: a few L2 round
-            // trips for the whole grid instead of one per 32 units
+            // 16 independent loads per lane in flight before any store, of 4 lengths each
+            // when lens is 16-byte aligned: one L2 round trip for up to 2048 units
             constexpr int BATCH = 16;
             const int cu = units / HS;  // cache units
-            for (int u0 = 0; u0 < cu; u0 += 32 * BATCH) {
+            const int n4 = (reinterpret_cast<uintptr_t>(a.lens) & 15u) == 0 ? cu / 4 : 0;
+            int4 *l4 = reinterpret_cast<int4 *>(a.lens);
+            for (int i0 = 0; i0 < n4; i0 += 32 * BATCH) {
+                int4 L[BATCH];
+#pragma unroll
+                for (int k = 0; k < BATCH; ++k) {
+                    const int i = i0 + 32 * k + lane;
+                    L[k] = i < n4 ? __ldcg(l4 + i) : make_int4(-1, -1, -1, -1);
+                }
+#pragma unroll
+                for (int k = 0; k < BATCH; ++k) {
+                    const int i = i0 + 32 * k + lane;
+                    if (i < n4) {
+                        int4 v = L[k];
+                        v.x += unit_ok(v.x, a.L_cap, a.append) ? 1 : 0;
+                        v.y += unit_ok(v.y, a.L_cap, a.append) ? 1 : 0;
+                        v.z += unit_ok(v.z, a.L_cap, a.append) ? 1 : 0;
+                        v.w += unit_ok(v.w, a.L_cap, a.append) ? 1 : 0;
+                        l4[i] = v;
+                    }
+                }
+            }
+            for (int u0 = 4 * n4; u0 < cu; u0 += 32 * BATCH) {  // the rest (or all) one length at a time
                 int L[BATCH];
 #pragma unroll
                 for (int k = 0; k < BATCH; ++k) {
@@ -847,11 +1009,21 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         }
         __syncwarp();
         if (lane == 0) {
-            a.counters[0] = 0;
-            a.counters[1] = 0;
+            *reinterpret_cast<unsigned long long *>(a.counters) = 0ull;
             if (rs >= 0) *a.slot = (rs + 1) % a.slots;  // every warp has read the row by now
         }
     }
+}
+
+// The launch's queries into the window ring after the SIMT decode: chunk c (16 bytes)
+// of query row c / ch goes to row *slot of that head's `slots` rows.
+__global__ void qring_copy(const uint4 *__restrict__ q, uint4 *__restrict__ qring, long long n16, int ch, int slots,
+                           const long long *slot)
+{
+    const long long s = *slot;
+    if (s < 0 || s >= slots) return;  // the decode has reported the slot
+    for (long long c = (long long)blockIdx.x * blockDim.x + threadIdx.x; c < n16; c += (long long)gridDim.x * blockDim.x)
+        qring[(c / ch * slots + s) * ch + c % ch] = q[c];
 }
 
 // The ring slot's advance after the SIMT decode (its CTAs have no last-warp step).
@@ -871,7 +1043,7 @@ static bool encode_cache_map(CUtensorMap *map, const void *base, unsigned long l
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
                           int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
                           const DecodeWs &ws, unsigned *err, cudaStream_t s, float *ring, int slots,
-                          long long *slot)
+                          long long *slot, void *qring)
 {
     DecodeArgs a;
     a.K = kv.k;
@@ -898,6 +1070,8 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.slot = slot;
     a.slots = slots;
     a.nq = (long long)kv.n_layers * kv.B * kv.H_q;
+    a.qring = ring ? qring : nullptr;
+    a.q_bytes = kv.dtype == RECO_F32 ? 4 : 2;
     const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
     // partial slots: two per warp of the grid
     const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.part_slots;
@@ -942,6 +1116,14 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || !ring) return e;
+    if (a.qring) {
+        const int ch = kv.d * a.q_bytes / 16;
+        const long long n16 = a.nq * ch;
+        const unsigned blocks = (unsigned)std::min<long long>((n16 + 255) / 256, 4LL * device_sm_count());
+        qring_copy<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4 *>(q), reinterpret_cast<uint4 *>(a.qring), n16,
+                                          ch, slots, slot);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     ring_advance<<<1, 1, 0, s>>>(slot, slots);
     return cudaGetLastError();
 }

@@ -83,7 +83,7 @@ cudaError_t launch_compact(const reco_kv &kv, const int32_t *kept_idx, int32_t *
 cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, const void *v_new,
                           int32_t *lens, float scale, void *out, reco_dtype out_dtype, float *lse,
                           const DecodeWs &ws, unsigned *err, cudaStream_t s, float *ring = nullptr,
-                          int slots = 0, long long *slot = nullptr);
+                          int slots = 0, long long *slot = nullptr, void *qring = nullptr);
 cudaError_t launch_penalty(float *logits, int B, int V, const int32_t *ids, int n_ids,
                            const float *rewards, float tau_l, float tau_h, float beta, float *beta_out,
                            unsigned *err, cudaStream_t s);

@@ -4,14 +4,16 @@
 // step reward (float32 compares); Eq. 4 subtracts it from the logit of every
 // reflection token, in place.  R is a set: an id listed twice is penalised once.
 //
-// sample_segments + sample_pick: Eq. 3-4 and then one draw per row from softmax of the
-// penalised logits (Sec. 3.3, temperature 1) by inversion at a caller-supplied uniform.
+// sample_cluster (or sample_segments + sample_pick for unaligned or very long rows):
+// Eq. 3-4 and then one draw per row from softmax of the penalised logits (Sec. 3.3,
+// temperature 1) by inversion at a caller-supplied uniform.
 //
 // ppl_rows + ppl_finish: Eq. 5 log p(x_t) = z[x_t] - logsumexp(z) per answer row
 // (one CTA per row, one streaming pass with an online max/sum), then per sequence
 // PPL = exp(-mean log p) and the Eq. 6 stop flag PPL <= tau_p.
 #include "common.cuh"
 #include "internal.h"
+#include "tma.cuh"
 
 namespace reco {
 
@@ -282,10 +284,248 @@ __global__ void __launch_bounds__(NT) sample_pick(const float *__restrict__ logi
     if (tid == 0) tokens[b] = tok >= 0 ? tok : last_tok;
 }
 
+// ---------------------------------------------------------------- penalty + sampling in one launch
+// One cluster of C <= 8 CTAs per row, for rows of 16-byte aligned float32 logits (V a
+// multiple of 4) of at most C * kSampleClusterRecs records of kSampleRec tokens.  CTA r
+// of the cluster brings records [r * rpc, (r + 1) * rpc) of its row into shared memory
+// with bulk copies, applies the Eq. 4 penalty to the ids inside them (in shared memory
+// and in place in global memory, the same correctly rounded subtract as above), and
+// writes each record's log2-domain (max, sum) into CTA 0's shared memory.  After a
+// cluster barrier CTA 0 draws exactly as sample_pick does, with records in place of
+// segments, reading the chosen record from its owner CTA's shared memory; a second
+// cluster barrier keeps every CTA's shared memory alive until that read is done.  The
+// row is read from HBM once and no workspace is used.
+constexpr int kSampleRec = 1024;          // tokens per record
+constexpr int kSampleClusterRecs = 48;    // records per CTA at most (192 KB of shared memory)
+constexpr int kSampleCluster = 8;         // CTAs per row at most (the portable cluster size)
+constexpr long long kSampleSpin = 1LL << 24;  // bounded wait on the bulk copies (about a second)
+
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void st_cluster_f2(uint32_t addr, float x, float y)
+{
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(x), "f"(y) : "memory");
+}
+
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr)
+{
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+
+// All threads of all CTAs of the cluster; shared-memory writes before it (local or
+// remote) are visible to every CTA after it.
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Untiled bulk copy global -> shared (both 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(dst), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+template <int NT>
+__global__ void __launch_bounds__(NT) sample_cluster(float *__restrict__ logits, int V, int rpc,
+                                                     const int32_t *__restrict__ ids, int n_ids,
+                                                     const float *__restrict__ rewards, float tau_l, float tau_h,
+                                                     float beta, float *__restrict__ beta_out,
+                                                     const float *__restrict__ uniforms,
+                                                     int32_t *__restrict__ tokens, unsigned *err)
+{
+    constexpr int NWARP = NT / 32;
+    constexpr int SR = (kSampleCluster * kSampleClusterRecs + NT - 1) / NT;  // records per thread (pick)
+    constexpr int PER = kSampleRec / NT;                                     // tokens per thread (pick)
+    constexpr int RL = kSampleRec / 32;                                      // tokens per lane (records)
+    static_assert(PER == 4, "the pick reads one float4 of the chosen record per thread");
+    extern __shared__ __align__(128) float sm_z[];  // [rpc * kSampleRec] this CTA's part of the row
+    __shared__ float2 sm_rec[NT * SR];               // (max, sum) of every record of the row (CTA 0)
+    __shared__ int sm_ids[kIdsShared];
+    __shared__ float sm_w[NWARP];
+    __shared__ float sm_f[1];
+    __shared__ int sm_i[2];
+    __shared__ __align__(8) uint64_t bar;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const uint32_t r = cluster_rank();
+    const int b = blockIdx.y;
+    const int nrec = (V + kSampleRec - 1) / kSampleRec;
+    const int lo = (int)r * rpc * kSampleRec;  // first token held here
+    const int hi = min(V, lo + rpc * kSampleRec);
+    const int nr = hi > lo ? (hi - lo + kSampleRec - 1) / kSampleRec : 0;  // records held here
+    const uint32_t bar_a = smem_addr(&bar), z_a = smem_addr(sm_z);
+    if (tid == 0) {
+        mbar_init(bar_a, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        fence_async_shared();
+    }
+    __syncthreads();
+    wait_prior_grid();
+    float *z = logits + (size_t)b * V;
+    if (tid == 0 && nr > 0) {  // the copies run while the ids and the reward load
+        const uint32_t bytes = (uint32_t)(hi - lo) * 4u;
+        mbar_expect_tx(bar_a, bytes);
+        for (uint32_t off = 0; off < bytes; off += 16384u)
+            bulk_load(z_a + off, z + lo + off / 4u, min(16384u, bytes - off), bar_a);
+    }
+    const float v = rewards[b];
+    const float bi = (v <= tau_l) ? 0.f : ((v >= tau_h) ? beta : beta * 0.5f);
+    if (r == 0 && tid == 0 && beta_out) beta_out[b] = bi;
+    const bool staged = stage_ids(ids, n_ids, sm_ids);
+    bool landed = true;
+    if (nr > 0) {
+        landed = mbar_wait_bounded(bar_a, 0, kSampleSpin);
+        if (!landed && tid == 0) raise_error(err, ERR_INTERNAL);
+    }
+    for (int i = tid; i < n_ids; i += NT) {
+        const int id = staged ? sm_ids[i] : ids[i];
+        if (id < 0 || id >= V) {
+            if (b == 0 && r == 0) raise_error(err, ERR_ID);
+            continue;
+        }
+        if (id < lo || id >= hi || bi == 0.f || !landed) continue;
+        if (!seen_before(ids, sm_ids, staged, i, id)) {
+            const float pz = __fsub_rn(sm_z[id - lo], bi);
+            sm_z[id - lo] = pz;
+            z[id] = pz;
+        }
+    }
+    __syncthreads();  // the penalised records are visible to the whole CTA
+
+    // one warp per record: its log2-domain (max, sum), into CTA 0's table
+    const uint32_t rec0 = cluster_addr(smem_addr(sm_rec), 0);
+    for (int k = wid; k < nr; k += NWARP) {
+        float y[RL];
+        float m = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < RL; ++i) {
+            const int j = k * kSampleRec + i * 32 + lane;
+            y[i] = lo + j < hi ? sm_z[j] * kLog2e : -INFINITY;
+            m = fmaxf(m, y[i]);
+        }
+        float s = 0.f;
+        if (m != -INFINITY) {
+#pragma unroll
+            for (int i = 0; i < RL; ++i) s += fast_exp2(y[i] - m);  // -inf terms add 0
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+            const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+            lse_merge(m, s, m2, s2);
+        }
+        if (lane == 0) st_cluster_f2(rec0 + (uint32_t)((int)r * rpc + k) * 8u, m, s);
+    }
+    cluster_sync();
+
+    if (r == 0) {  // uniform across the CTA
+        float2 q[SR];
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < SR; ++k) {
+            const int g = tid * SR + k;
+            q[k] = g < nrec ? sm_rec[g] : make_float2(-INFINITY, 0.f);
+            M = fmaxf(M, q[k].x);
+        }
+        M = warp_max(M);
+        if (lane == 0) sm_w[wid] = M;
+        __syncthreads();
+        M = sm_w[0];
+        for (int w2 = 1; w2 < NWARP; ++w2) M = fmaxf(M, sm_w[w2]);
+        __syncthreads();
+        if (M == -INFINITY) {  // no token has mass
+            if (tid == 0) tokens[b] = -1;
+        } else {
+            float w[SR];
+            float zsum = 0.f;
+#pragma unroll
+            for (int k = 0; k < SR; ++k) {
+                w[k] = q[k].y > 0.f ? q[k].y * fast_exp2(q[k].x - M) : 0.f;
+                zsum += w[k];
+            }
+            zsum = warp_sum(zsum);
+            if (lane == 0) sm_w[wid] = zsum;
+            __syncthreads();
+            float Z = 0.f;
+            for (int w2 = 0; w2 < NWARP; ++w2) Z += sm_w[w2];
+            __syncthreads();
+            const float u = uniforms[b];
+            const float T = u != u ? u : fmaxf(u, 0.f) * Z;  // a NaN draw finds no crossing
+            float before;
+            int last_rec;
+            int rec = find_crossing<NT, SR>(w, tid * SR, T, sm_w, sm_i, sm_f, before, last_rec);
+            const bool found = rec >= 0;
+            if (!found) rec = last_rec;
+            const float Tr = found ? fmaxf(T - before, 0.f) : INFINITY;
+            // the chosen record, from the shared memory of the CTA that holds it
+            const int first = rec * kSampleRec + tid * PER;
+            const float4 zz = ld_cluster_f4(
+                cluster_addr(z_a + (uint32_t)((rec % rpc) * kSampleRec + tid * PER) * 4u, (uint32_t)(rec / rpc)));
+            const float zv[PER] = {zz.x, zz.y, zz.z, zz.w};
+            float p[PER];
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                const float y = first + k < V ? zv[k] * kLog2e : -INFINITY;
+                p[k] = y == -INFINITY ? 0.f : fast_exp2(y - M);
+            }
+            float before2;
+            int last_tok;
+            const int tok = find_crossing<NT, PER>(p, first, Tr, sm_w, sm_i, sm_f, before2, last_tok);
+            if (tid == 0) tokens[b] = tok >= 0 ? tok : last_tok;
+        }
+    }
+    cluster_sync();  // CTA 0 has read the chosen record
+}
+
 cudaError_t launch_penalty_sample(float *logits, int B, int V, const int32_t *ids, int n_ids, const float *rewards,
                                   float tau_l, float tau_h, float beta, const float *uniforms, int32_t *tokens,
                                   float *beta_out, float2 *part, unsigned *err, cudaStream_t s)
 {
+    const int nrec = (V + kSampleRec - 1) / kSampleRec;
+    const int C = nrec < kSampleCluster ? nrec : kSampleCluster;
+    const int rpc = (nrec + C - 1) / C;
+    if ((V & 3) == 0 && ((uintptr_t)logits & 15u) == 0 && rpc <= kSampleClusterRecs) {
+        const size_t smem = (size_t)rpc * kSampleRec * sizeof(float);
+        cudaError_t e = cudaFuncSetAttribute(sample_cluster<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSampleClusterRecs * kSampleRec * (int)sizeof(float));
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(C, B);
+        cfg.blockDim = dim3(256);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[2];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = C;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 2;
+        return cudaLaunchKernelEx(&cfg, sample_cluster<256>, logits, V, rpc, ids, n_ids, rewards, tau_l, tau_h, beta,
+                                  beta_out, uniforms, tokens, err);
+    }
+    // other rows: two launches through the workspace
     const int nseg = (V + kSampleSeg - 1) / kSampleSeg;
     cudaError_t e = launch_pdl(sample_segments<256>, dim3(nseg, B), dim3(256), 0, s, logits, V, nseg, ids, n_ids,
                                rewards, tau_l, tau_h, beta, beta_out, part, err);

@@ -70,7 +70,7 @@ def lib():
     L.reco_select_topm.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_compact.argtypes = [kvp, vp, vp, vp, i32, vp]
     L.reco_decode_attn.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, vp, sz, vp]
-    L.reco_decode_attn_ring.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, i32, vp, vp, sz, vp]
+    L.reco_decode_attn_ring.argtypes = [kvp, vp, vp, vp, vp, f32, vp, i32, vp, i32, vp, vp, vp, sz, vp]
     L.reco_reflect_penalty.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp]
     L.reco_penalty_sample.argtypes = [vp, i32, i32, vp, i32, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp]
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
@@ -213,14 +213,21 @@ def reco_decode_attn(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, lse,
                                ws.numel(), _stream(stream)))
 
 
-def reco_decode_attn_ring(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, ring, slot, ws, stream=None):
+def reco_decode_attn_ring(kv: reco_kv, q, k_new, v_new, lens, scale: float, out, ring, slot, ws, stream=None,
+                          q_ring=None):
     """reco_decode_attn with the lse written into ring rows slot and slot + S (ring [2 * S, n]
-    float32) and slot (one-element int64 device tensor) advanced, on the device."""
+    float32) and slot (one-element int64 device tensor) advanced, on the device; with
+    q_ring ([Ly, B, Hq, S, d], q's dtype) each head's query also goes to its row slot."""
     if ring.dim() < 2 or ring.shape[0] % 2:
         raise ValueError("ring must have an even number of rows")
+    S = int(ring.shape[0]) // 2
+    if q_ring is not None and (q_ring.dim() != 5 or q_ring.shape[3] != S or q_ring.dtype != q.dtype
+                               or tuple(q_ring.shape[:3]) + (q_ring.shape[4],) != tuple(q.shape)
+                               or not q_ring.is_contiguous()):
+        raise ValueError("q_ring must be a contiguous [Ly, B, Hq, S, d] tensor of q's dtype")
     _ok(lib().reco_decode_attn_ring(ctypes.byref(kv), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(lens), float(scale),
-                                    _ptr(out), _dtype_code(out.dtype), _ptr(ring), int(ring.shape[0]) // 2,
-                                    _ptr(slot), _ptr(ws), ws.numel(), _stream(stream)))
+                                    _ptr(out), _dtype_code(out.dtype), _ptr(ring), S, _ptr(slot), _ptr(q_ring),
+                                    _ptr(ws), ws.numel(), _stream(stream)))
 
 
 def reco_reflect_penalty(logits, ids, rewards, tau_l=0.4, tau_h=0.8, beta=4.0, beta_out=None,

@@ -15,10 +15,11 @@ When a sequence completes a step it receives a reward v_i (Sec. 3.1), and
     keep = L, which skips their scoring and leaves them untouched;
   * if v_{i-1} >= tau_h and v_i >= tau_h, the answer probe runs (Eq. 5-6) and a
     sequence that passes PPL <= tau_p stops and leaves the batch.
-Eq. 2's observation window is the queries of the last w decoded tokens.  The lse each
-decode returns is kept in a device ring; when none of the sequences compressed at a
-boundary was compressed within its window, those lse are the window rows' normalisers
-and the scores take one pass over K (reco_score_cache_lse), else two (reco_score_cache).
+Eq. 2's observation window is the queries of the last w decoded tokens.  Those queries
+and the lse each decode returns are kept in device rings of w slots, written by every
+token; when none of the sequences compressed at a boundary was compressed within its
+window, those lse are the window rows' normalisers and the scores take one pass over K
+(reco_score_cache_lse), else two (reco_score_cache).
 Budget base L (the paper is silent on repeated compression): reading "A" uses the
 current cache length, reading "B" the full uncompressed length so far (the keep
 count is then capped at the current length).  Lengths are tracked on the host, so
@@ -27,7 +28,8 @@ the loop needs no device read-back except the stop flags of a probe.
 With use_graph, a token's decode, penalty, draw and lse push are one captured CUDA
 graph over static input buffers (captured again whenever the batch shrinks), so the
 per-token host work is one graph launch (with an input pool, the graph also gathers
-the token's inputs).
+the token's inputs); a boundary uploads keep counts and rewards and launches the
+scoring and selection, with no host-side gather of the window.
 """
 from __future__ import annotations
 
@@ -133,8 +135,8 @@ class TraceEvents:
 class Trace:
     def __init__(self, spec: TraceSpec, device="cuda", out_dtype=torch.float32, input_pool: int = 0,
                  use_graph: bool = False):
-        """input_pool > 0: per-token inputs are drawn once for that many tokens and reused
-        cyclically (timing runs); 0: every token draws its own seeded inputs.
+        """input_pool = w (the window): per-token inputs are drawn once for w tokens and
+        reused cyclically (timing runs); 0: every token draws its own seeded inputs.
         use_graph: the per-token decode + penalty runs as a captured CUDA graph."""
         self.spec = spec
         self.input_pool = input_pool
@@ -180,15 +182,18 @@ class Trace:
                     t = int(self.ends[sq][k])
                     if t < spec.generated and r[k - 1] >= np.float32(wl.tau_h) and r[k] >= np.float32(wl.tau_h):
                         self._answers[(t, sq)] = self._answer(t, sq)
-        # The decode's lse of the last R tokens (ring row t % R holds token t's, mirrored in
-        # row t % R + R so that any w consecutive tokens are contiguous rows; with an input
-        # pool R is its size, so one device counter selects both) and, per active
-        # sequence, how many tokens were decoded since its last compression: Eq. 2's window
-        # rows are those tokens' queries, and their lse are the rows' normalisers while the
-        # cache has not been compressed since they were decoded.
-        self.R = input_pool if input_pool else 64
-        if self.R < wl.w:
-            raise ValueError(f"input_pool {input_pool} is shorter than the window {wl.w}")
+        # The window ring: the queries (q_win, slot t % w of every head's w rows) and the
+        # decode's lse (ring row t % w, mirrored in row t % w + w) of the last w tokens, kept
+        # by every token on the device; one device counter (slot_dev = t % w) also selects
+        # the input-pool slot.  Per active sequence, `since` counts the tokens decoded since
+        # its last compression: Eq. 2's window rows are those tokens' queries, and their lse
+        # are the rows' normalisers while the cache has not been compressed since they were
+        # decoded.  In that one-pass form Eq. 2 sums the same rows whatever their order (every
+        # candidate key precedes the whole window), so the ring is scored in slot order; the
+        # two-pass form (causal row normalisers) gets the window rotated into token order.
+        self.R = wl.w
+        if input_pool and input_pool != self.R:
+            raise ValueError(f"input_pool must be 0 or the window w = {self.R} (one counter selects both)")
         self.lse_ring = torch.zeros((2 * self.R, wl.layers, spec.batch, wl.h_q), dtype=torch.float32,
                                     device=device)
         self.slot_dev = torch.zeros(1, dtype=torch.long, device=device)
@@ -257,20 +262,10 @@ class Trace:
             return self._slot_view(t % self.input_pool, 4)
         return self._sel(self._token_draws(t), 0)
 
-    def _window(self, toks, slots, rows):
-        """Eq. 2's window queries of the sequences at batch positions `rows`: their queries of
-        the tokens `toks` (the last w decoded; input-pool slots `slots`), written into those
-        rows of q_win [Ly, B, Hq, w, d] (the other rows are not read by a masked scoring)."""
-        # moved as 16-byte elements (a query row of d values is d * es / 16 of them)
-        if self._apool is not None:
-            off, nb, dt, shape = self._slot_meta[0]
-            Q = self._apool[:, off:off + nb].view(torch.complex128).view(self.input_pool, *shape[:-1], -1)
-            qs = Q.permute(0, 2, 1, 3, 4)[slots[:, None], rows[None, :]]  # [w, k, Ly, Hq, d/8], one gather
-        else:
-            qs = torch.stack([self._sel(self._token_inputs(tt)[0]) for tt in toks]).permute(0, 2, 1, 3, 4)[:, rows]
-            qs = qs.contiguous().view(torch.complex128)
-        self.q_win.view(torch.complex128).permute(1, 3, 0, 2, 4)[rows] = qs.permute(1, 0, 2, 3, 4)
-        return self.q_win
+    def _window_in_token_order(self, t: int):
+        """q_win rotated so that row k holds the query of token t - w + 1 + k (the two-pass
+        scoring's causal row normalisers depend on the row's position)."""
+        return torch.roll(self.q_win, shifts=-((t + 1) % self.R), dims=3)
 
     # ---------------------------------------------------------------- plumbing
     def _active_pool(self):
@@ -331,7 +326,9 @@ class Trace:
         self.last_comp = [self.last_comp[i] for i in keep_pos]
         self.since = [self.since[i] for i in keep_pos]
         self.lse_ring = self.lse_ring.index_select(2, idx).contiguous()
+        q_win = self.q_win.index_select(1, idx)
         self._rebuild()
+        self.q_win.copy_(q_win)
 
     def _capture(self, t: int):
         """Static input/output buffers and one CUDA graph of a token's decode + penalty.
@@ -367,10 +364,10 @@ class Trace:
                 # fewer nanoseconds than 8-byte ones for the same bytes
                 torch.index_select(self._apool.view(torch.complex128), 0, self.slot_dev,
                                    out=self.g_in.view(torch.complex128).view(1, -1))
-            # the token's lse goes straight into the ring, and the decode advances the slot
-            # (the next token's pool slot)
+            # the token's lse and queries go straight into the window rings, and the decode
+            # advances the slot (the next token's pool slot)
             reco.reco_decode_attn_ring(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,
-                                       self.lse_ring, self.slot_dev, self.ws_decode)
+                                       self.lse_ring, self.slot_dev, self.ws_decode, q_ring=self.q_win)
             if self.g_logits is not None:
                 reco.reco_penalty_sample(self.g_logits, self.ids, self.g_rw, self.g_u, self.g_tok, self.ws_sample,
                                          wl.tau_l, wl.tau_h, wl.beta)
@@ -378,11 +375,11 @@ class Trace:
         self._slot_t = t
         self.graph = g
 
-    def _put_small(self, keep, extra=()):
-        """Upload keep counts, the active sequences' current rewards and `extra` ints into
-        g_small in one copy; returns the device view written."""
+    def _put_small(self, keep):
+        """Upload keep counts and the active sequences' current rewards into g_small in one
+        copy; returns the device view written."""
         rw = np.asarray([self.current_reward(s) for s in self.active], np.float32).view(np.int32)
-        vals = np.concatenate([np.asarray(keep, np.int32), rw, np.asarray(extra, np.int32)])
+        vals = np.concatenate([np.asarray(keep, np.int32), rw])
         return self.staging.put(vals, torch.int32, out=self.g_small[:len(vals)])
 
     def current_reward(self, s: int) -> float:
@@ -413,7 +410,7 @@ class Trace:
         q, kn, vn = self.active_inputs(t)
         out = torch.empty(q.shape, dtype=self.out_dtype, device=self.device)
         reco.reco_decode_attn_ring(self.kv, q, kn, vn, self.lens_dev, wl.scale(), out, self.lse_ring, self.slot_dev,
-                                   self.ws_decode)
+                                   self.ws_decode, q_ring=self.q_win)
         lse = self.lse_ring[t % self.R]
         self._slot_t = t + 1
         logits = None
@@ -472,32 +469,28 @@ class Trace:
             q_win = None
             if info:
                 comp = [self.pos[s] for s, _, _ in info]
-                # Eq. 2's window: the queries of the last w decoded tokens (ring / pool slots)
-                toks = range(t - wl.w + 1, t + 1)
-                extra = [tt % self.R for tt in toks] + comp
                 if self.use_graph and self.graph is not None:
-                    # keep counts, the new rewards and the window's slots and rows together
-                    small = self._put_small(keep, extra)
-                    keep_dev, idx = small[:self.B], small[2 * self.B:]
+                    keep_dev = self._put_small(keep)[:self.B]  # with the new rewards
                 else:
-                    small = self.staging.put(list(keep) + extra, torch.int32)
-                    keep_dev, idx = small[:self.B], small[self.B:]
-                slots, rows = idx[:wl.w], idx[wl.w:]
-                q_win = self._window(toks, slots, rows)
+                    keep_dev = self.staging.put(list(keep), torch.int32)
                 # only the sequences compressed now are scored (keep == L skips the rest)
                 if all(self.since[i] >= wl.w for i in comp):
                     # every window token was decoded on the cache as it is now, so the lse
-                    # its decode returned is its row's normaliser: one pass over K
-                    s0 = (t - wl.w + 1) % self.R
-                    reco.reco_score_cache_lse(self.kv, q_win, self.lens_dev, self.lse_ring[s0:s0 + wl.w], wl.w,
+                    # its decode returned is its row's normaliser: one pass over K, with the
+                    # rings' rows in slot order
+                    q_win = self.q_win
+                    reco.reco_score_cache_lse(self.kv, q_win, self.lens_dev, self.lse_ring[:wl.w], wl.w,
                                               wl.pool, wl.scale(), self.scores, self.ws_score, keep=keep_dev)
                     ev.lse_scorings += 1
                 else:
+                    q_win = self._window_in_token_order(t)
                     reco.reco_score_cache(self.kv, q_win, self.lens_dev, wl.w, wl.pool, wl.scale(), self.scores,
                                           self.ws_score, keep=keep_dev)
                     ev.two_pass_scorings += 1
                 reco.reco_select_compact(self.kv, self.scores, self.lens_dev, keep_dev, wl.w, self.kept,
                                          self.ws_select)
+                if on_boundary and q_win is self.q_win:
+                    q_win = self._window_in_token_order(t)  # the caller sees token order
             if on_boundary:
                 on_boundary(t, self, done, keep, q_win)
             for i in range(len(keep)):

@@ -164,8 +164,8 @@ def test_penalty_sample_validates_before_launch(L):
 
 
 def test_split_select_compact_and_ring_decode_validate_before_launch(L):
-    """reco_select_topm, reco_compact and reco_decode_attn_ring reject bad arguments on the
-    host, before any launch."""
+    """reco_select_topm, reco_compact and reco_decode_attn_ring (also a q_ring off a 16-byte
+    boundary) reject bad arguments on the host, before any launch."""
     kv = _kv()
     vp = ctypes.c_void_p
     ws = vp(256 * 1000)
@@ -190,11 +190,12 @@ def test_split_select_compact_and_ring_decode_validate_before_launch(L):
     assert st == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
     st = L.reco_compact(ctypes.byref(kv), vp(16), vp(16), vp(16), 101, None)
     assert st == reco.RECO_EINVAL and b"window" in L.reco_last_error()
-    dec = lambda kv_, ring, slots, slot: L.reco_decode_attn_ring(  # noqa: E731
-        ctypes.byref(kv_), vp(16), None, None, vp(16), 0.1, vp(16), 0, ring, slots, slot, ws, 10, None)
+    dec = lambda kv_, ring, slots, slot, q_ring=None: L.reco_decode_attn_ring(  # noqa: E731
+        ctypes.byref(kv_), vp(16), None, None, vp(16), 0.1, vp(16), 0, ring, slots, slot, q_ring, ws, 10, None)
     assert dec(kv, vp(16), 0, vp(16)) == reco.RECO_EINVAL and b"slots" in L.reco_last_error()
     assert dec(kv, None, 4, vp(16)) == reco.RECO_EINVAL
     assert dec(kv, vp(16), 4, vp(20)) == reco.RECO_EINVAL and b"aligned" in L.reco_last_error()
+    assert dec(kv, vp(16), 4, vp(16), vp(24)) == reco.RECO_EINVAL and b"q_ring" in L.reco_last_error()
     # past its own checks it applies reco_decode_attn's (here: the workspace is too short)
     assert dec(kv, vp(16), 4, vp(16)) == reco.RECO_EINVAL and b"workspace" in L.reco_last_error()
     assert dec(_kv(H_q=34, H_kv=2), vp(16), 4, vp(16)) == reco.RECO_EUNSUPPORTED

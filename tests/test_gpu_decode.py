@@ -164,6 +164,24 @@ def test_tma_path_unit_limit(shape):
     _check(wl, lens, True)
 
 
+@pytest.mark.parametrize("shape,top", [((28, 14, 28, 4), 255), ((28, 32, 28, 4), 255), ((2, 3, 7, 1), 255),
+                                       ((8, 4, 32, 2), 255), ((28, 14, 28, 4), 256)])
+def test_short_units_sorted_and_dealt_whole(shape, top):
+    """Units of at most 16 blocks after the append are sorted by length and dealt whole to the
+    warps in snake order: fewer units than warps, between one and two per warp, more than two,
+    two halves of 16 heads per KV head, and (top 256, 17 blocks with the append) the switch back
+    to the contiguous deal.  Units without keys (no append) and of one key are among them."""
+    layers, batch, h_q, h_kv = shape
+    wl = W.WORKLOADS["7b"].reduced(layers=layers, batch=batch, h_q=h_q, h_kv=h_kv, L=300, decode_steps=2)
+    rng = np.random.default_rng(layers * batch + top)
+    lens = rng.integers(0, top + 1, (layers, batch, h_kv)).astype(np.int32)
+    flat = lens.reshape(-1)
+    flat[:3] = [0, 1, top]
+    flat[-2:] = [0, top]
+    _check(wl, lens, False)  # units of length 0 have no keys: zero output, lse -inf
+    _check(wl, lens, True, steps=2)
+
+
 @pytest.mark.parametrize("h_q,h_kv", [(16, 2), (12, 1), (9, 3)])
 def test_bf16_decode_more_than_8_heads_per_kv_head(h_q, h_kv):
     """G = 8, 12, 3 ... and 16, 12, 9 heads per KV head: the TMA path takes a unit of more than

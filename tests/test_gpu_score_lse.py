@@ -189,7 +189,8 @@ def test_lse_push_ring_and_slot():
 def test_decode_attn_ring_matches_decode_then_push(dtype, h_q, h_kv, L):
     """reco_decode_attn_ring is reco_decode_attn followed by reco_lse_push: the same outputs,
     cache and lengths, the lse in ring rows slot and slot + S (bit-exact), the slot advanced
-    (with a wrap-around), on the TMA path (bf16, G 7), the SIMT path (G 16, and float32)."""
+    (with a wrap-around), each head's query in its row slot of q_ring (the other rows
+    untouched), on the TMA path (bf16, G 7), the SIMT path (G 16, and float32)."""
     wl = W.WORKLOADS["7b"].reduced(layers=2, batch=3, h_q=h_q, h_kv=h_kv, L=L, decode_steps=4, dtype=dtype)
     Ka, Va = W.make_cache(wl, DEV, canary=False)
     Kb, Vb = Ka.clone(), Va.clone()
@@ -201,24 +202,30 @@ def test_decode_attn_ring_matches_decode_then_push(dtype, h_q, h_kv, L):
     S, n = 3, wl.layers * wl.batch * wl.h_q
     ring_a, ring_b = torch.zeros((2 * S, n), device=DEV), torch.zeros((2 * S, n), device=DEV)
     slot_a, slot_b = torch.tensor([1], dtype=torch.int64, device=DEV), torch.tensor([1], dtype=torch.int64, device=DEV)
+    q_ring = torch.full((wl.layers, wl.batch, wl.h_q, S, wl.d), -3.0, dtype=wl.torch_dtype, device=DEV)
+    q_ref = q_ring.clone()
     for s in range(4):
         q, kn, vn = W.make_decode_step(wl, s, DEV)
         oa, ob = torch.empty(q.shape, device=DEV), torch.empty(q.shape, device=DEV)
         lse = torch.empty(q.shape[:3], device=DEV)
         reco.reco_decode_attn(kva, q, kn, vn, la, wl.scale(), oa, lse, wsa)
         reco.reco_lse_push(lse, ring_a, slot_a)
-        reco.reco_decode_attn_ring(kvb, q, kn, vn, lb, wl.scale(), ob, ring_b, slot_b, wsb)
+        q_ref[:, :, :, (1 + s) % S] = q
+        reco.reco_decode_attn_ring(kvb, q, kn, vn, lb, wl.scale(), ob, ring_b, slot_b, wsb, q_ring=q_ring)
         reco.reco_check()
         assert torch.equal(oa, ob) and torch.equal(la, lb)
         assert torch.equal(ring_a, ring_b) and int(slot_b.item()) == (2 + s) % S
+        assert torch.equal(q_ring.view(torch.uint8), q_ref.view(torch.uint8))
     assert torch.equal(Ka.view(torch.uint8), Kb.view(torch.uint8))
     # an out-of-range slot: no ring row written, slot kept, the error word set
     before = ring_b.clone()
     slot_b.fill_(S)
     q, kn, vn = W.make_decode_step(wl, 9, DEV)
-    reco.reco_decode_attn_ring(kvb, q, None, None, lb, wl.scale(), torch.empty(q.shape, device=DEV), ring_b, slot_b, wsb)
+    reco.reco_decode_attn_ring(kvb, q, None, None, lb, wl.scale(), torch.empty(q.shape, device=DEV), ring_b, slot_b, wsb,
+                               q_ring=q_ring)
     with pytest.raises(reco.RecoError) as e:
         reco.reco_check()
     assert e.value.status == reco.RECO_EDEVICE
     assert torch.equal(ring_b, before) and int(slot_b.item()) == S
+    assert torch.equal(q_ring.view(torch.uint8), q_ref.view(torch.uint8))
     reco.reco_check()

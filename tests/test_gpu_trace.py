@@ -157,7 +157,7 @@ def _run(spec, track=None, decode_every=1, use_graph=False, input_pool=0):
     return tr, rep, ev
 
 
-@pytest.mark.parametrize("use_graph,input_pool", [(False, 0), (True, 0), (True, 64)])
+@pytest.mark.parametrize("use_graph,input_pool", [(False, 0), (True, 0), (True, 32)])
 def test_trace_reading_A_reduced(use_graph, input_pool):
     # tau_h 0.6 so that this seed's Beta(2,2) rewards trigger probes (4 probes, 3 stops)
     base = W.WORKLOADS["7b"].reduced(layers=2, vocab=5000, tau_h=0.6)

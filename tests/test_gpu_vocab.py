@@ -173,6 +173,22 @@ def test_penalty_sample_ragged_vocab_and_edge_draws(V):
     _sample_case(z, ids_np, np.array([1.0, 0.5, 0.0, 0.9, 1.0, 0.3], np.float32), u_np, max_inexact=1)
 
 
+@pytest.mark.parametrize("V,offset", [(9216, 0), (152064, 0), (393216, 0), (393220, 0), (152064, 1)])
+def test_penalty_sample_one_launch_limits(V, offset):
+    """Rows drawn in one launch (a cluster per row): CTAs of the cluster left without
+    records (V 9216), the largest row (V 393216, 48 records per CTA), then one record past
+    it and a row off a 16-byte boundary, both drawn through the workspace."""
+    rng = np.random.default_rng(V + offset)
+    B = 3
+    buf = torch.from_numpy((rng.standard_normal(B * V + offset) * 2).astype(np.float32)).to(DEV)
+    z = buf[offset:].view(B, V)
+    ids_np = rng.choice(V, 40, replace=False).astype(np.int32)
+    ids_np[:8] = np.arange(V - 8, V)  # ids in the last record
+    ids_np[8] = ids_np[9]  # a repeated id: one subtraction
+    u_np = np.array([0.3, np.float32(1 - 2 ** -24), 0.0], np.float32)
+    _sample_case(z, ids_np, np.array([1.0, 0.5, 0.9], np.float32), u_np, max_inexact=1)
+
+
 def test_penalty_sample_masked_tokens_and_empty_rows():
     rng = np.random.default_rng(33)
     B, V = 8, 9000
