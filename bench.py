@@ -724,7 +724,7 @@ def run_trace(args):
         spec.generated = args.generated
     use_graph = not args.no_graph
     warm = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=32, use_graph=use_graph)
-    warm.run(max_tokens=128)
+    warm.run(max_tokens=320)  # past the first probe (and its stop): every kernel and path warm
     torch.cuda.synchronize()
     tr = trace.Trace(spec, "cuda", torch.bfloat16, input_pool=32, use_graph=use_graph)
     torch.cuda.synchronize()

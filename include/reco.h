@@ -169,6 +169,17 @@ reco_status reco_score_cache_lse(const reco_kv *kv, const void *q_win, const int
  *          nothing and sets the device error word.                              */
 reco_status reco_lse_push(const float *lse, int64_t n, float *ring, int slots, int64_t *slot, cudaStream_t stream);
 
+/* Step-loop utility, not a step of the method: copies row *index of src, a
+ * [rows][row_bytes] device array, into dst, with the row chosen on the device, so a
+ * captured graph copies a different row on every replay (e.g. the next token's inputs
+ * from a pool, selected by the same counter the decode advances).
+ *   src   : [rows][row_bytes] (device, 16-byte aligned), row_bytes a multiple of 16
+ *   index : int64 (device, read only); a value outside [0, rows) copies nothing and
+ *           sets the device error word
+ *   dst   : [row_bytes] (device, 16-byte aligned, written)                        */
+reco_status reco_copy_row(const void *src, int64_t rows, int64_t row_bytes, const int64_t *index, void *dst,
+                          cudaStream_t stream);
+
 /* Top-m selection and in-place compaction (Sec. 3.2: keep the m_i best tokens,
  * the latest w always retained; compress the L cached tokens down to m_i).
  * For unit (layer, b, h) with L = lens[unit] and m = keep[b]:

@@ -292,6 +292,21 @@ reco_status reco_lse_push(const float *lse, int64_t n, float *ring, int slots, i
     return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_lse_push launch");
 }
 
+reco_status reco_copy_row(const void *src, int64_t rows, int64_t row_bytes, const int64_t *index, void *dst,
+                          cudaStream_t stream)
+{
+    if (rows < 1 || row_bytes < 16 || row_bytes % 16) return fail(RECO_EINVAL, "need rows >= 1 and row_bytes a positive multiple of 16");
+    if (!src || !index || !dst) return fail(RECO_EINVAL, "NULL src, index or dst");
+    if (!al16(src) || !al16(dst) || ((uintptr_t)index & 7u))
+        return fail(RECO_EINVAL, "src and dst must be 16-byte aligned, index 8-byte aligned");
+    unsigned *err;
+    reco_status st = error_word(&err);
+    if (st != RECO_OK) return st;
+    cudaError_t e = reco::launch_copy_row(src, (long long)rows, (long long)row_bytes,
+                                          reinterpret_cast<const long long *>(index), dst, err, stream);
+    return e == cudaSuccess ? RECO_OK : cuda_fail(e, "reco_copy_row launch");
+}
+
 reco_status reco_select_compact(const reco_kv *kv, const float *scores, int32_t *lens, const int32_t *keep, int w,
                                 int32_t *kept_idx, void *ws, size_t ws_bytes, cudaStream_t stream)
 {

@@ -69,6 +69,8 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
 cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep,
                              const float *row_lse, int w, int pool, float scale, float *scores, const ScoreWs &ws,
                              unsigned *err, cudaStream_t s);
+cudaError_t launch_copy_row(const void *src, long long rows, long long row_bytes, const long long *index, void *dst,
+                            unsigned *err, cudaStream_t s);
 cudaError_t launch_lse_push(const float *lse, long n, float *ring, int slots, long long *slot, unsigned *err,
                             cudaStream_t s);
 cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_t *lens,

@@ -12,6 +12,8 @@
 // This file holds the SIMT passes used for float32 caches (and any shape the tensor-
 // core passes do not cover), the combine and pool kernels, and the launcher;
 // score_tc.cu holds the bf16 tensor-core (tcgen05) passes.
+#include <algorithm>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -420,6 +422,47 @@ cudaError_t launch_lse_push(const float *lse, long n, float *ring, int slots, lo
                             cudaStream_t s)
 {
     cudaError_t e = launch_pdl(lse_push_kernel, dim3(1), dim3(1024), 0, s, lse, n, ring, slots, slot, err);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Row *index of a [rows][n16] array of 16-byte chunks into dst, for captured step loops
+// whose input row is chosen on the device: a grid of a few CTAs per SM, eight independent
+// 16-byte loads per thread in flight before its stores.
+__global__ void __launch_bounds__(256) copy_row_kernel(const uint4 *__restrict__ src, long long rows, long long n16,
+                                                     const long long *__restrict__ index, uint4 *__restrict__ dst,
+                                                     unsigned *err)
+{
+    wait_prior_grid();  // the index (and the destination's readers) belong to earlier kernels
+    const long long r = *index;
+    if (r < 0 || r >= rows) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) raise_error(err, ERR_INTERNAL);
+        return;
+    }
+    const uint4 *row = src + r * n16;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long i0 = (long long)blockIdx.x * blockDim.x + threadIdx.x; i0 < n16; i0 += 8 * stride) {
+        uint4 v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const long long i = i0 + k * stride;
+            if (i < n16) v[k] = ld_stream_u4(row + i);
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const long long i = i0 + k * stride;
+            if (i < n16) dst[i] = v[k];
+        }
+    }
+}
+
+cudaError_t launch_copy_row(const void *src, long long rows, long long row_bytes, const long long *index, void *dst,
+                            unsigned *err, cudaStream_t s)
+{
+    const long long n16 = row_bytes / 16;
+    const long long want = (n16 + 256LL * 8 - 1) / (256LL * 8);
+    const unsigned grid = (unsigned)std::max(1LL, std::min(want, 4LL * device_sm_count()));
+    cudaError_t e = launch_pdl(copy_row_kernel, dim3(grid), dim3(256), 0, s, reinterpret_cast<const uint4 *>(src), rows,
+                               n16, index, reinterpret_cast<uint4 *>(dst), err);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 

@@ -20,7 +20,7 @@ RECO_OP_SCORE, RECO_OP_SELECT, RECO_OP_DECODE, RECO_OP_PPL, RECO_OP_SAMPLE = ran
 
 EXPORTS = ("reco_retention_ratio", "reco_keep_count", "reco_penalty_band", "reco_probe_trigger",
            "reco_workspace_bytes", "reco_last_error", "reco_check", "reco_score_cache",
-           "reco_score_cache_lse", "reco_lse_push", "reco_select_compact", "reco_select_topm", "reco_compact",
+           "reco_score_cache_lse", "reco_lse_push", "reco_copy_row", "reco_select_compact", "reco_select_topm", "reco_compact",
            "reco_decode_attn", "reco_decode_attn_ring", "reco_reflect_penalty", "reco_penalty_sample", "reco_answer_ppl",
            "reco_answer_ppl_static")
 RECO_PPL_STATIC_MAX_ROWS = 65536
@@ -66,6 +66,7 @@ def lib():
     L.reco_score_cache.argtypes = [kvp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_score_cache_lse.argtypes = [kvp, vp, vp, vp, vp, i32, i32, f32, vp, vp, sz, vp]
     L.reco_lse_push.argtypes = [vp, ctypes.c_int64, vp, i32, vp, vp]
+    L.reco_copy_row.argtypes = [vp, ctypes.c_int64, ctypes.c_int64, vp, vp, vp]
     L.reco_select_compact.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_select_topm.argtypes = [kvp, vp, vp, vp, i32, vp, vp, sz, vp]
     L.reco_compact.argtypes = [kvp, vp, vp, vp, i32, vp]
@@ -76,7 +77,7 @@ def lib():
     L.reco_answer_ppl.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, sz, vp]
     L.reco_answer_ppl_static.argtypes = [vp, vp, vp, i32, i32, i32, f32, vp, vp, vp]
     for name in ("reco_retention_ratio", "reco_keep_count", "reco_workspace_bytes", "reco_check",
-                 "reco_score_cache", "reco_score_cache_lse", "reco_lse_push", "reco_select_compact",
+                 "reco_score_cache", "reco_score_cache_lse", "reco_lse_push", "reco_copy_row", "reco_select_compact",
                  "reco_select_topm", "reco_compact",
                  "reco_decode_attn", "reco_decode_attn_ring", "reco_reflect_penalty", "reco_penalty_sample",
                  "reco_answer_ppl",
@@ -180,6 +181,18 @@ def reco_lse_push(lse, ring, slot, stream=None):
     if ring.dim() < 2 or ring[0].numel() != n or ring.shape[0] % 2:
         raise ValueError("ring must have an even number of rows of lse.numel() floats")
     _ok(lib().reco_lse_push(_ptr(lse), n, _ptr(ring), int(ring.shape[0]) // 2, _ptr(slot), _stream(stream)))
+
+
+def reco_copy_row(src, index, dst, stream=None):
+    """dst = src[index] on the device: src [rows, ...] (each row a multiple of 16 bytes),
+    index a one-element int64 device tensor, dst a tensor of one row's bytes."""
+    rows = src.shape[0]
+    row_bytes = src[0].numel() * src.element_size()
+    if not src.is_contiguous() or not dst.is_contiguous() or dst.numel() * dst.element_size() != row_bytes:
+        raise ValueError("src and dst must be contiguous and dst one row of src")
+    if index.dtype != torch.int64 or index.numel() != 1:
+        raise ValueError("index must be a one-element int64 tensor")
+    _ok(lib().reco_copy_row(_ptr(src), rows, row_bytes, _ptr(index), _ptr(dst), _stream(stream)))
 
 
 def reco_score_cache_lse(kv: reco_kv, q_win, lens, row_lse, w: int, pool_kernel: int, scale: float, scores, ws,

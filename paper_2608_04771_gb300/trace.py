@@ -360,10 +360,9 @@ class Trace:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="relaxed"):
             if self._apool is not None:
-                # 16-byte elements (every part is a multiple of 256 bytes): a quarter
-                # fewer nanoseconds than 8-byte ones for the same bytes
-                torch.index_select(self._apool.view(torch.complex128), 0, self.slot_dev,
-                                   out=self.g_in.view(torch.complex128).view(1, -1))
+                # the token's packed inputs: pool row slot_dev (every part a multiple of
+                # 256 bytes), selected on the device
+                reco.reco_copy_row(self._apool, self.slot_dev, self.g_in)
             # the token's lse and queries go straight into the window rings, and the decode
             # advances the slot (the next token's pool slot)
             reco.reco_decode_attn_ring(self.kv, self.g_q, self.g_kn, self.g_vn, self.lens_dev, wl.scale(), self.g_out,

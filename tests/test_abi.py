@@ -201,6 +201,18 @@ def test_split_select_compact_and_ring_decode_validate_before_launch(L):
     assert dec(_kv(H_q=34, H_kv=2), vp(16), 4, vp(16)) == reco.RECO_EUNSUPPORTED
 
 
+def test_copy_row_validates_before_launch(L):
+    vp = ctypes.c_void_p
+    assert L.reco_copy_row(vp(256), 0, 64, vp(8), vp(256), None) == reco.RECO_EINVAL
+    assert L.reco_copy_row(vp(256), 4, 72 + 1, vp(8), vp(256), None) == reco.RECO_EINVAL
+    assert L.reco_copy_row(vp(256), 4, 0, vp(8), vp(256), None) == reco.RECO_EINVAL
+    assert L.reco_copy_row(vp(264), 4, 64, vp(8), vp(256), None) == reco.RECO_EINVAL
+    assert b"aligned" in L.reco_last_error()
+    assert L.reco_copy_row(vp(256), 4, 64, vp(12), vp(256), None) == reco.RECO_EINVAL
+    assert L.reco_copy_row(vp(256), 4, 64, None, vp(256), None) == reco.RECO_EINVAL
+    assert L.reco_copy_row(vp(256), 4, 64, vp(8), vp(260), None) == reco.RECO_EINVAL
+
+
 def test_decode_workspace_counts_a_ticket_per_half_unit_above_8_heads(L):
     """A unit of more than 8 query heads per KV head runs as two units on the tensor path, with
     a merge ticket each: the workspace holds one more int per unit."""

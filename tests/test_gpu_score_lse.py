@@ -229,3 +229,45 @@ def test_decode_attn_ring_matches_decode_then_push(dtype, h_q, h_kv, L):
     assert torch.equal(ring_b, before) and int(slot_b.item()) == S
     assert torch.equal(q_ring.view(torch.uint8), q_ref.view(torch.uint8))
     reco.reco_check()
+
+
+def test_copy_row_selects_the_row_on_the_device():
+    """reco_copy_row copies row *index, read on the device: plain calls, a captured graph whose
+    index moves between replays, a row of several grid passes, and out-of-range indices (nothing
+    copied, the device error word set)."""
+    rng = np.random.default_rng(11)
+    src = torch.from_numpy(rng.integers(0, 256, (5, 4096 * 3 + 16 * 7), dtype=np.uint8)).to(DEV)
+    dst = torch.zeros(src.shape[1], dtype=torch.uint8, device=DEV)
+    idx = torch.zeros(1, dtype=torch.int64, device=DEV)
+    for r in (0, 4, 2):
+        idx.fill_(r)
+        reco.reco_copy_row(src, idx, dst)
+        reco.reco_check()
+        assert torch.equal(dst, src[r])
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        reco.reco_copy_row(src, idx, dst, s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            reco.reco_copy_row(src, idx, dst, s)
+    torch.cuda.synchronize()
+    for r in (3, 1):
+        idx.fill_(r)
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(dst, src[r])
+    big = torch.from_numpy(rng.integers(0, 256, (2, 24 << 20), dtype=np.uint8)).to(DEV)  # several passes
+    dbig = torch.zeros(big.shape[1], dtype=torch.uint8, device=DEV)
+    idx.fill_(1)
+    reco.reco_copy_row(big, idx, dbig)
+    reco.reco_check()
+    assert torch.equal(dbig, big[1])
+    before = dst.clone()
+    for bad in (5, -1):
+        idx.fill_(bad)
+        reco.reco_copy_row(src, idx, dst)
+        with pytest.raises(reco.RecoError) as e:
+            reco.reco_check()
+        assert e.value.status == reco.RECO_EDEVICE
+        assert torch.equal(dst, before)
+    reco.reco_check()
