@@ -599,6 +599,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             }
     };
 
+    // K and V rows are read once per launch: evict them first, so they do not displace the
+    // queries, the outputs, the partials or the next kernels' inputs from L2 (a medium cache,
+    // 1792 units of 200-400 rows, went from 62.1 to 56.6 us; the 7B-class launch 1.5% faster)
+    const uint64_t kv_policy = l2_evict_first_policy();
     // ---- block stream: lane 0 keeps up to S blocks in flight, running from the current
     // item into the next one (grabbed one item ahead) so no refill bubble opens between
     // items; the warp consumes blocks in issue order.
@@ -630,8 +634,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             mbar_expect_tx(bar, STAGE);
 #pragma unroll
             for (int hh = 0; hh < HALVES; ++hh) {
-                tma_load_2d(dst + hh * TILE, &tmK, 64 * hh, y, bar);
-                tma_load_2d(dst + (HALVES + hh) * TILE, &tmV, 64 * hh, y, bar);
+                tma_load_2d_hint(dst + hh * TILE, &tmK, 64 * hh, y, bar, kv_policy);
+                tma_load_2d_hint(dst + (HALVES + hh) * TILE, &tmV, 64 * hh, y, bar, kv_policy);
             }
         }
         ++pblk;
