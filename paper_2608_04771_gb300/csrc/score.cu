@@ -136,6 +136,39 @@ __global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, 
     rowb[i] = m + log2f(z);
 }
 
+// The units a masked call scores, in ascending order (one CTA; a ballot scan per
+// blockDim.x units), and their count.
+__device__ __forceinline__ void unit_list_block(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap,
+                                                int units, int32_t *__restrict__ ulist, int32_t *__restrict__ ucount)
+{
+    __shared__ int warp_n[32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int base = 0;
+    for (int u0 = 0; u0 < units; u0 += blockDim.x) {
+        const int u = u0 + threadIdx.x;
+        const bool take = u < units && !mask.skip(u, lens[u], w, L_cap);
+        const unsigned bal = __ballot_sync(0xffffffffu, take);
+        if (lane == 0) warp_n[wid] = __popc(bal);
+        __syncthreads();
+        int off = base, tot = 0;
+        for (int k = 0; k < nw; ++k) {
+            off += k < wid ? warp_n[k] : 0;
+            tot += warp_n[k];
+        }
+        if (take) ulist[off + __popc(bal & ((1u << lane) - 1u))] = u;
+        base += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *ucount = base;
+}
+
+__global__ void __launch_bounds__(1024) score_unit_list(const int32_t *__restrict__ lens, ScoreMask mask, int w,
+                                                        int L_cap, int units, int32_t *__restrict__ ulist,
+                                                        int32_t *__restrict__ ucount)
+{
+    unit_list_block(lens, mask, w, L_cap, units, ulist, ucount);
+}
+
 // Row normalisers from log-sum-exps the decode already produced (Eq. 2 with one pass over
 // K).  Window row (g, t) is query head g of the token at position L - w + t; when that
 // token was decoded the cache held exactly the keys j <= L - w + t that Eq. 2's causal
@@ -145,8 +178,13 @@ __global__ void score_combine(const int32_t *__restrict__ lens, ScoreMask mask, 
 // normaliser at +inf, so the row adds nothing to the scores.
 __global__ void score_rowb_from_lse(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap, int R, int G,
                                     int Hq, int Hkv, long rows_q, const float *__restrict__ row_lse,
-                                    float *__restrict__ rowb, long units, unsigned *err)
+                                    float *__restrict__ rowb, long units, int32_t *__restrict__ ulist,
+                                    int32_t *__restrict__ ucount, unsigned *err)
 {
+    if (ulist != nullptr && blockIdx.x == gridDim.x - 1) {  // the extra block: the units a masked call scores
+        unit_list_block(lens, mask, w, L_cap, (int)units, ulist, ucount);
+        return;
+    }
     const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= units * R) return;
     const long u = i / R;
@@ -278,6 +316,29 @@ __global__ void __launch_bounds__(128) score_colsum_simt(
 }
 
 // Max-pool over the clipped window [j - pool/2, j + pool/2] within [0, L-w).
+// score_pool over the units of a masked call's list only: CTAs (blockIdx.x: a 256-key
+// chunk) walk the list, so the units left out cost no CTAs.
+__global__ void score_pool_list(const float *__restrict__ raw, const int32_t *__restrict__ lens,
+                                const int32_t *__restrict__ ulist, const int32_t *__restrict__ ucount, int w,
+                                int L_cap, int pool, float *__restrict__ scores)
+{
+    const int n = *ucount;
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    const int half = pool / 2;
+    for (int k = blockIdx.y; k < n; k += gridDim.y) {
+        const long u = ulist[k];
+        const int L = lens[u];
+        if (L < w || L > L_cap) continue;
+        const int nc = L - w;
+        if (j >= nc) continue;
+        const int lo = max(0, j - half), hi = min(nc - 1, j + half);
+        const float *rp = raw + u * L_cap;
+        float m = rp[lo];
+        for (int i = lo + 1; i <= hi; ++i) m = fmaxf(m, rp[i]);
+        scores[u * L_cap + j] = m;
+    }
+}
+
 __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restrict__ lens, ScoreMask mask, int w,
                            int L_cap, int pool, float *__restrict__ scores)
 {
@@ -295,32 +356,6 @@ __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restr
     scores[u * L_cap + j] = m;
 }
 
-// The units a masked call scores, in ascending order (one CTA; a ballot scan per
-// 1024 units), and their count.
-__global__ void __launch_bounds__(1024) score_unit_list(const int32_t *__restrict__ lens, ScoreMask mask, int w,
-                                                        int L_cap, int units, int32_t *__restrict__ ulist,
-                                                        int32_t *__restrict__ ucount)
-{
-    __shared__ int warp_n[32];
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    int base = 0;
-    for (int u0 = 0; u0 < units; u0 += blockDim.x) {
-        const int u = u0 + threadIdx.x;
-        const bool take = u < units && !mask.skip(u, lens[u], w, L_cap);
-        const unsigned bal = __ballot_sync(0xffffffffu, take);
-        if (lane == 0) warp_n[wid] = __popc(bal);
-        __syncthreads();
-        int off = base, tot = 0;
-        for (int k = 0; k < nw; ++k) {
-            off += k < wid ? warp_n[k] : 0;
-            tot += warp_n[k];
-        }
-        if (take) ulist[off + __popc(bal & ((1u << lane) - 1u))] = u;
-        base += tot;
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) *ucount = base;
-}
 
 cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
                                   float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
@@ -381,6 +416,23 @@ static cudaError_t score_simt_any(const reco_kv &kv, const void *q_win, const in
                                                 pass1);
 }
 
+// Max-pooling of the raw scores into `scores`: over the unit list when the call built one
+// (a masked tensor-core call), else one CTA per (unit, 256-key chunk).
+static cudaError_t launch_pool(const reco_kv &kv, const int32_t *lens, ScoreMask mask, bool listed, int w, int pool,
+                               float *scores, const ScoreWs &ws, cudaStream_t s)
+{
+    const long units = (long)kv.n_layers * kv.B * kv.H_kv;
+    const unsigned chunks = (unsigned)((kv.L_cap + 255) / 256);
+    if (listed) {
+        const long walkers = std::max(1L, 8L * device_sm_count() / (long)chunks);
+        score_pool_list<<<dim3(chunks, (unsigned)std::min(units, std::min(walkers, 65535L))), 256, 0, s>>>(
+            ws.raw, lens, ws.ulist, ws.ucount, w, kv.L_cap, pool, scores);
+    } else {
+        score_pool<<<dim3(chunks, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap, pool, scores);
+    }
+    return cudaGetLastError();
+}
+
 cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *lens, const int32_t *keep, int w,
                          int pool, float scale, float *scores, const ScoreWs &ws, unsigned *err, cudaStream_t s)
 {
@@ -389,7 +441,8 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
     const ScoreMask mask{keep, kv.B, kv.H_kv};
     cudaError_t e = cudaSuccess;
     bool used_tc = false;
-    if (kv.dtype == RECO_BF16 && score_tc_supported(kv, w)) {
+    const bool tc = kv.dtype == RECO_BF16 && score_tc_supported(kv, w);
+    if (tc) {
         // tensor-core passes: (unit list) -> pass 1 -> combine -> pass 2
         if (keep) {
             score_unit_list<<<1, 1024, 0, s>>>(lens, mask, w, kv.L_cap, (int)units, ws.ulist, ws.ucount);
@@ -413,9 +466,7 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
         e = score_simt_any(kv, q_win, lens, mask, w, c2, ws, err, s, true);
         if (e != cudaSuccess) return e;
     }
-    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,
-                                                                            pool, scores);
-    return cudaGetLastError();
+    return launch_pool(kv, lens, mask, tc && keep, w, pool, scores, ws, s);
 }
 
 cudaError_t launch_lse_push(const float *lse, long n, float *ring, int slots, long long *slot, unsigned *err,
@@ -477,13 +528,11 @@ cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t
     const long rows_q = (long)kv.n_layers * kv.B * kv.H_q;
     const bool tc = kv.dtype == RECO_BF16 && score_tc_supported(kv, w);
     cudaError_t e;
-    if (tc && keep) {
-        score_unit_list<<<1, 1024, 0, s>>>(lens, mask, w, kv.L_cap, (int)units, ws.ulist, ws.ucount);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    score_rowb_from_lse<<<(unsigned)((units * R + 255) / 256), 256, 0, s>>>(lens, mask, w, kv.L_cap, R, G, kv.H_q,
-                                                                           kv.H_kv, rows_q, row_lse, ws.rowb, units,
-                                                                           err);
+    // the row normalisers, and (a masked tensor-core call) the unit list from one extra block
+    const bool listed = tc && keep;
+    const unsigned blocks = (unsigned)((units * R + 255) / 256) + (listed ? 1u : 0u);
+    score_rowb_from_lse<<<blocks, 256, 0, s>>>(lens, mask, w, kv.L_cap, R, G, kv.H_q, kv.H_kv, rows_q, row_lse, ws.rowb,
+                                               units, listed ? ws.ulist : nullptr, listed ? ws.ucount : nullptr, err);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     bool used = false;
     if (tc) {
@@ -494,9 +543,7 @@ cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t
         e = score_simt_any(kv, q_win, lens, mask, w, c2, ws, err, s, false);
         if (e != cudaSuccess) return e;
     }
-    score_pool<<<dim3((kv.L_cap + 255) / 256, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap,
-                                                                            pool, scores);
-    return cudaGetLastError();
+    return launch_pool(kv, lens, mask, tc && keep, w, pool, scores, ws, s);
 }
 
 }  // namespace reco
