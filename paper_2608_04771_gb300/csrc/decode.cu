@@ -686,6 +686,14 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         const __nv_bfloat16 *vn = a.append ? reinterpret_cast<const __nv_bfloat16 *>(a.v_new) + (long)pu * D : nullptr;
         const long qrow0 = lb * a.Hq + (long)h * a.G + cur.hp * GS;
         const int row0 = pu * a.L_cap;  // first tensor-map row of this unit
+        // this lane's 16-byte chunk of the appended row (K for lanes < D/8, V for the next
+        // D/8), loaded now so that neither the stage patch nor the cache write below waits
+        // on global memory
+        uint4 app = make_uint4(0, 0, 0, 0);
+        if (Lapp >= k0 && Lapp < k1 && lane < 2 * (D / 8)) {
+            const bool isv = lane >= D / 8;
+            app = *reinterpret_cast<const uint4 *>((isv ? vn : kn) + (isv ? lane - D / 8 : lane) * 8);
+        }
 
         // start this item's copies before the wait on its query registers below
         __syncwarp();
@@ -729,8 +737,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
                     const int rr = Lapp - kb;
                     const bool isv = lane >= HALVES * 8;
                     const int ch = isv ? lane - HALVES * 8 : lane;
-                    const uint4 val = *reinterpret_cast<const uint4 *>((isv ? vn : kn) + ch * 8);
-                    sts_u4((isv ? Vs : Ks) + (ch >> 3) * TILE + swz(rr, ch & 7), val);
+                    sts_u4((isv ? Vs : Ks) + (ch >> 3) * TILE + swz(rr, ch & 7), app);
                 }
                 __syncwarp();
             }
@@ -825,7 +832,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
             const bool isv = lane >= D / 8;
             const int pc = isv ? lane - D / 8 : lane;
             __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(isv ? a.V : a.K) + ((long)row0 + Lapp) * D + pc * 8;
-            *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>((isv ? vn : kn) + pc * 8);
+            *reinterpret_cast<uint4 *>(dst) = app;
         }
 
         const int q0 = 2 * c, q1 = 2 * c + 1;

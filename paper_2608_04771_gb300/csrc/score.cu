@@ -166,6 +166,7 @@ __global__ void __launch_bounds__(1024) score_unit_list(const int32_t *__restric
                                                         int L_cap, int units, int32_t *__restrict__ ulist,
                                                         int32_t *__restrict__ ucount)
 {
+    wait_prior_grid();
     unit_list_block(lens, mask, w, L_cap, units, ulist, ucount);
 }
 
@@ -181,6 +182,7 @@ __global__ void score_rowb_from_lse(const int32_t *__restrict__ lens, ScoreMask 
                                     float *__restrict__ rowb, long units, int32_t *__restrict__ ulist,
                                     int32_t *__restrict__ ucount, unsigned *err)
 {
+    wait_prior_grid();  // lens and the ring rows may come from the previous kernels
     if (ulist != nullptr && blockIdx.x == gridDim.x - 1) {  // the extra block: the units a masked call scores
         unit_list_block(lens, mask, w, L_cap, (int)units, ulist, ucount);
         return;
@@ -322,6 +324,7 @@ __global__ void score_pool_list(const float *__restrict__ raw, const int32_t *__
                                 const int32_t *__restrict__ ulist, const int32_t *__restrict__ ucount, int w,
                                 int L_cap, int pool, float *__restrict__ scores)
 {
+    wait_prior_grid();  // the raw scores and the list come from the previous kernels
     const int n = *ucount;
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     const int half = pool / 2;
@@ -342,6 +345,7 @@ __global__ void score_pool_list(const float *__restrict__ raw, const int32_t *__
 __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restrict__ lens, ScoreMask mask, int w,
                            int L_cap, int pool, float *__restrict__ scores)
 {
+    wait_prior_grid();  // the raw scores come from the previous kernel
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     const long u = blockIdx.y;
     const int L = lens[u];
@@ -425,10 +429,14 @@ static cudaError_t launch_pool(const reco_kv &kv, const int32_t *lens, ScoreMask
     const unsigned chunks = (unsigned)((kv.L_cap + 255) / 256);
     if (listed) {
         const long walkers = std::max(1L, 8L * device_sm_count() / (long)chunks);
-        score_pool_list<<<dim3(chunks, (unsigned)std::min(units, std::min(walkers, 65535L))), 256, 0, s>>>(
-            ws.raw, lens, ws.ulist, ws.ucount, w, kv.L_cap, pool, scores);
+        const unsigned ys = (unsigned)std::min(units, std::min(walkers, 65535L));
+        cudaError_t e = launch_pdl(score_pool_list, dim3(chunks, ys), dim3(256), 0, s, (const float *)ws.raw, lens,
+                                   (const int32_t *)ws.ulist, (const int32_t *)ws.ucount, w, kv.L_cap, pool, scores);
+        if (e != cudaSuccess) return e;
     } else {
-        score_pool<<<dim3(chunks, (unsigned)units), 256, 0, s>>>(ws.raw, lens, mask, w, kv.L_cap, pool, scores);
+        cudaError_t e = launch_pdl(score_pool, dim3(chunks, (unsigned)units), dim3(256), 0, s, (const float *)ws.raw, lens,
+                                   mask, w, kv.L_cap, pool, scores);
+        if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
 }
@@ -445,8 +453,9 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
     if (tc) {
         // tensor-core passes: (unit list) -> pass 1 -> combine -> pass 2
         if (keep) {
-            score_unit_list<<<1, 1024, 0, s>>>(lens, mask, w, kv.L_cap, (int)units, ws.ulist, ws.ucount);
-            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+            e = launch_pdl(score_unit_list, dim3(1), dim3(1024), 0, s, lens, mask, w, kv.L_cap, (int)units, ws.ulist,
+                           ws.ucount);
+            if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
         }
         e = launch_score_tc_pass1(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used_tc);
         if (e != cudaSuccess) return e;
@@ -531,8 +540,9 @@ cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t
     // the row normalisers, and (a masked tensor-core call) the unit list from one extra block
     const bool listed = tc && keep;
     const unsigned blocks = (unsigned)((units * R + 255) / 256) + (listed ? 1u : 0u);
-    score_rowb_from_lse<<<blocks, 256, 0, s>>>(lens, mask, w, kv.L_cap, R, G, kv.H_q, kv.H_kv, rows_q, row_lse, ws.rowb,
-                                               units, listed ? ws.ulist : nullptr, listed ? ws.ucount : nullptr, err);
+    e = launch_pdl(score_rowb_from_lse, dim3(blocks), dim3(256), 0, s, lens, mask, w, kv.L_cap, R, G, kv.H_q, kv.H_kv,
+                   rows_q, row_lse, ws.rowb, units, listed ? ws.ulist : nullptr, listed ? ws.ucount : nullptr, err);
+    if (e != cudaSuccess) return e;
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     bool used = false;
     if (tc) {

@@ -290,9 +290,6 @@ __global__ void __launch_bounds__(Pass1Cfg<D, MT, N, EG>::THREADS, 1)
     __shared__ int abort_sh;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
-    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
-    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
     const uint32_t raw0 = smem_addr(smem_raw);
     const uint32_t base = (raw0 + 1023u) & ~1023u;
     const uint32_t Qs = base;                // MT x HALVES x QBOX
@@ -320,6 +317,12 @@ __global__ void __launch_bounds__(Pass1Cfg<D, MT, N, EG>::THREADS, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
     volatile int *abort_flag = &abort_sh;
+    // everything above runs while the previous kernel drains; from here on its outputs
+    // (the unit list, the row normalisers, the window queries) are read
+    wait_prior_grid();
+    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
+    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
 
     if (warp == 0) {
         if (lane == 0) {  // producer: queries when the unit changes, then the chunk's K tiles
@@ -533,9 +536,6 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
     __shared__ float cpart[S][EG][128];  // per tile slot: each group's partial column sums
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
-    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
-    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
     const int NW = NQ / NP;                     // columns of one piece
     const int stride = (NW + 31) & ~31;         // TMEM columns between regions
     const uint32_t raw0 = smem_addr(smem_raw);
@@ -570,6 +570,12 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
     volatile int *abort_flag = &abort_sh;
+    // everything above runs while the previous kernel drains; from here on its outputs
+    // (the unit list, the row normalisers, the window queries) are read
+    wait_prior_grid();
+    const int n_it = ucount ? *ucount * n_chunks : n_items;  // items of the scored units
+    const int i_begin = (int)((long long)blockIdx.x * n_it / gridDim.x);
+    const int i_end = (int)((long long)(blockIdx.x + 1) * n_it / gridDim.x);
 
     if (warp == 0) {
         if (lane == 0) {  // producer
@@ -787,11 +793,11 @@ static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t
     if (e != cudaSuccess) return e;
     const int n_items = (int)(units * nch);
     const int grid = min(n_items, device_sm_count());
-    score_rowstats_tc<D, MT, N, EG><<<grid, C::THREADS, C::SMEM, s>>>(
-        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, nch, n_items, masked ? ws.ulist : nullptr,
-        masked ? ws.ucount : nullptr, c2, ws.part_m, ws.part_z, err);
+    e = launch_pdl(score_rowstats_tc<D, MT, N, EG>, dim3(grid), dim3(C::THREADS), C::SMEM, s, mq, mk, lens, w,
+                   kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, nch, n_items, masked ? ws.ulist : nullptr,
+                   masked ? ws.ucount : nullptr, c2, ws.part_m, ws.part_z, err);
     *ok = true;
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <int D>
@@ -845,11 +851,11 @@ static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t
     if (e != cudaSuccess) return e;
     const int n_items = (int)(units * nch);
     const int grid = min(n_items, device_sm_count());
-    score_colsum_tc<D><<<grid, 128 + 128 * kP2Groups, smem, s>>>(
-        mq, mk, lens, w, kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, ps.NQ, ps.NP, ps.NR, NS, nch, n_items,
-        masked ? ws.ulist : nullptr, masked ? ws.ucount : nullptr, c2, ws.rowb, ws.raw, err);
+    e = launch_pdl(score_colsum_tc<D>, dim3(grid), dim3(128 + 128 * kP2Groups), smem, s, mq, mk, lens, w,
+                   kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, ps.NQ, ps.NP, ps.NR, NS, nch, n_items,
+                   masked ? ws.ulist : nullptr, masked ? ws.ucount : nullptr, c2, ws.rowb, ws.raw, err);
     *ok = true;
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,

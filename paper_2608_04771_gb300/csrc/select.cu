@@ -89,6 +89,7 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
     __shared__ int tot[NT / 32 + 1];
     __shared__ uint32_t s_prefix;
     __shared__ int s_remaining;
+    wait_prior_grid();  // scores, lens and keep may come from the previous kernels
     for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
         const int tid = threadIdx.x, lane = tid & 31;
         const int b = (int)((u / Hkv) % B);
@@ -206,6 +207,7 @@ __global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__
     __shared__ int w_gt[NW], w_eq[NW];
     __shared__ uint32_t s_prefix;
     __shared__ int s_remaining;
+    wait_prior_grid();  // scores, lens and keep may come from the previous kernels
     for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
         const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
         const int b = (int)((u / Hkv) % B);
@@ -380,6 +382,7 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
 {
     constexpr int P = 8;  // 16-byte pieces per 128-byte slice
     constexpr int U = 2;  // rows per thread in one chunk
+    wait_prior_grid();    // kept indices, lens and the cache may belong to the previous kernels
     for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
         int lim;
         const int m = cnt.rows(u, err, lim);
@@ -433,6 +436,7 @@ __global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int3
 __global__ void compact_set_lens(int32_t *lens, const int32_t *__restrict__ keep, long units, int w, int B,
                                  int Hkv, int L_cap)
 {
+    wait_prior_grid();
     const long u = (long)blockIdx.x * blockDim.x + threadIdx.x;
     if (u >= units) return;
     const int L = lens[u], m = keep[(u / Hkv) % B];
@@ -467,12 +471,14 @@ static cudaError_t launch_select(const reco_kv &kv, const float *scores, const i
                                              (int)kSelectSmemKeys * (int)sizeof(uint32_t));
         if (e != cudaSuccess) return e;
         const unsigned grid = walk_grid(select_topm_smem<1024>, 1024, key_bytes, units, 1);
-        select_topm_smem<1024><<<grid, 1024, key_bytes, s>>>(scores, lens, lens_out, keep, w, kv.B, kv.H_kv, kv.L_cap,
-                                                             idx, count, units, err);
+        e = launch_pdl(select_topm_smem<1024>, dim3(grid), dim3(1024), key_bytes, s, scores, lens, lens_out, keep, w,
+                       kv.B, kv.H_kv, kv.L_cap, idx, count, units, err);
+        if (e != cudaSuccess) return e;
     } else {
         const unsigned grid = walk_grid(select_topm<1024>, 1024, 0, units, 1);
-        select_topm<1024><<<grid, 1024, 0, s>>>(scores, lens, lens_out, keep, w, kv.B, kv.H_kv, kv.L_cap, idx, count,
-                                                units, err);
+        cudaError_t e = launch_pdl(select_topm<1024>, dim3(grid), dim3(1024), 0, s, scores, lens, lens_out, keep, w,
+                                   kv.B, kv.H_kv, kv.L_cap, idx, count, units, err);
+        if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
 }
@@ -496,9 +502,9 @@ cudaError_t launch_select_compact(const reco_kv &kv, const float *scores, int32_
     int row_bytes;
     long units;
     const dim3 grid = compact_grid<CountFromSelect>(kv, row_bytes, units);
-    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, idx, CountFromSelect{ws.count, kv.L_cap}, kv.L_cap,
-                                      row_bytes, units, err);
-    return cudaGetLastError();
+    e = launch_pdl(compact_rows<CountFromSelect>, grid, dim3(256), 0, s, (char *)kv.k, (char *)kv.v, (const int32_t *)idx,
+                   CountFromSelect{ws.count, kv.L_cap}, kv.L_cap, row_bytes, units, err);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_select_only(const reco_kv &kv, const float *scores, const int32_t *lens, const int32_t *keep,
@@ -513,13 +519,13 @@ cudaError_t launch_compact(const reco_kv &kv, const int32_t *kept_idx, int32_t *
     int row_bytes;
     long units;
     const dim3 grid = compact_grid<CountFromKeep>(kv, row_bytes, units);
-    compact_rows<<<grid, 256, 0, s>>>((char *)kv.k, (char *)kv.v, kept_idx,
-                                      CountFromKeep{lens, keep, w, kv.B, kv.H_kv, kv.L_cap}, kv.L_cap, row_bytes,
-                                      units, err);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    compact_set_lens<<<(unsigned)((units + 255) / 256), 256, 0, s>>>(lens, keep, units, w, kv.B, kv.H_kv, kv.L_cap);
-    return cudaGetLastError();
+    cudaError_t e = launch_pdl(compact_rows<CountFromKeep>, grid, dim3(256), 0, s, (char *)kv.k, (char *)kv.v,
+                               kept_idx, CountFromKeep{lens, keep, w, kv.B, kv.H_kv, kv.L_cap}, kv.L_cap, row_bytes,
+                               units, err);
+    if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
+    e = launch_pdl(compact_set_lens, dim3((unsigned)((units + 255) / 256)), dim3(256), 0, s, lens, keep, units, w, kv.B,
+                   kv.H_kv, kv.L_cap);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace reco
