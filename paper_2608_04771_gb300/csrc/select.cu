@@ -46,6 +46,20 @@ SelectWs select_ws_layout(const reco_kv &kv, void *base)
 // Most candidates a unit may have for the shared-memory selection (192 KB of keys).
 constexpr int kSelectSmemKeys = 48 * 1024;
 
+// Units a walking CTA reads the headers of up front, all loads in flight together (a CTA
+// of a boundary call holds a few units, most of which it only skips or copies).
+constexpr int kWalkAhead = 64;
+
+// (L, m) of the CTA's units (at most kWalkAhead) into `lm`; the caller synchronises.
+__device__ __forceinline__ void walk_headers(int2 *lm, const int32_t *lens, const int32_t *keep, long units, int B,
+                                             int Hkv)
+{
+    for (int i = threadIdx.x; i < kWalkAhead; i += blockDim.x) {
+        const long u = blockIdx.x + (long)i * gridDim.x;
+        if (u < units) lm[i] = make_int2(lens[u], keep[(int)((u / Hkv) % B)]);
+    }
+}
+
 __device__ __forceinline__ uint32_t order_key(float f)
 {
     uint32_t u = __float_as_uint(f);
@@ -89,11 +103,14 @@ __global__ void __launch_bounds__(NT) select_topm(const float *__restrict__ scor
     __shared__ int tot[NT / 32 + 1];
     __shared__ uint32_t s_prefix;
     __shared__ int s_remaining;
+    __shared__ int2 s_lm[kWalkAhead];
     wait_prior_grid();  // scores, lens and keep may come from the previous kernels
-    for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
+    walk_headers(s_lm, lens, keep, units, B, Hkv);
+    __syncthreads();
+    int it = 0;
+    for (long u = blockIdx.x; u < units; u += gridDim.x, ++it) {  // a few CTAs per SM walk the units
         const int tid = threadIdx.x, lane = tid & 31;
-        const int b = (int)((u / Hkv) % B);
-        const int L = lens[u], m = keep[b];
+        const int L = s_lm[it].x, m = s_lm[it].y;  // the grid gives no CTA more than kWalkAhead units
         if (L < w || L > L_cap || m < w || m > L) {
             if (tid == 0) {
                 count[u] = 0;
@@ -207,11 +224,14 @@ __global__ void __launch_bounds__(NT) select_topm_smem(const float *__restrict__
     __shared__ int w_gt[NW], w_eq[NW];
     __shared__ uint32_t s_prefix;
     __shared__ int s_remaining;
+    __shared__ int2 s_lm[kWalkAhead];
     wait_prior_grid();  // scores, lens and keep may come from the previous kernels
-    for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
+    walk_headers(s_lm, lens, keep, units, B, Hkv);
+    __syncthreads();
+    int it = 0;
+    for (long u = blockIdx.x; u < units; u += gridDim.x, ++it) {  // a few CTAs per SM walk the units
         const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-        const int b = (int)((u / Hkv) % B);
-        const int L = lens[u], m = keep[b];
+        const int L = s_lm[it].x, m = s_lm[it].y;  // the grid gives no CTA more than kWalkAhead units
         if (L < w || L > L_cap || m < w || m > L) {
             if (tid == 0) {
                 count[u] = 0;
@@ -368,7 +388,7 @@ struct CountFromKeep {
         const int L = lens[u], m = keep[(u / Hkv) % B];
         lim = L;
         if (L < w || L > L_cap || m < w || m > L) {
-            if (blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0)
+            if (blockIdx.y == 0 && blockIdx.z == 0)  // one column slice reports (an atomic OR)
                 raise_error(err, (L < w || L > L_cap) ? ERR_LEN : ERR_KEEP);
             return 0;
         }
@@ -377,15 +397,25 @@ struct CountFromKeep {
 };
 
 template <class Count>
-__global__ void __launch_bounds__(256) compact_rows(char *K, char *V, const int32_t *__restrict__ idx_all,
+__global__ void __launch_bounds__(256, 8) compact_rows(char *K, char *V, const int32_t *__restrict__ idx_all,
                                                     Count cnt, int L_cap, int row_bytes, long units, unsigned *err)
 {
     constexpr int P = 8;  // 16-byte pieces per 128-byte slice
     constexpr int U = 2;  // rows per thread in one chunk
+    __shared__ int2 s_ml[kWalkAhead];  // (rows to move, source limit) of this CTA's units
     wait_prior_grid();    // kept indices, lens and the cache may belong to the previous kernels
-    for (long u = blockIdx.x; u < units; u += gridDim.x) {  // a few CTAs per SM walk the units
-        int lim;
-        const int m = cnt.rows(u, err, lim);
+    for (int i = threadIdx.x; i < kWalkAhead; i += blockDim.x) {
+        const long u = blockIdx.x + (long)i * gridDim.x;
+        if (u < units) {
+            int lim;
+            const int m = cnt.rows(u, err, lim);
+            s_ml[i] = make_int2(m, lim);
+        }
+    }
+    __syncthreads();
+    int it = 0;
+    for (long u = blockIdx.x; u < units; u += gridDim.x, ++it) {  // a few CTAs per SM walk the units
+        const int m = s_ml[it].x, lim = s_ml[it].y;  // the grid gives no CTA more than kWalkAhead units
         if (m == 0) continue;
         char *base = (blockIdx.y == 0 ? K : V) + u * (long)L_cap * row_bytes;
         const int32_t *idx = idx_all + u * L_cap;
@@ -455,7 +485,8 @@ static unsigned walk_grid(F fn, int threads, size_t smem, long units, int per_un
         (void)cudaGetLastError();
         per_sm = 1;
     }
-    const long ctas = std::max(1L, (long)per_sm * device_sm_count() / per_unit);
+    long ctas = std::max(1L, (long)per_sm * device_sm_count() / per_unit);
+    ctas = std::max(ctas, (units + kWalkAhead - 1) / kWalkAhead);  // at most kWalkAhead units per CTA
     return (unsigned)std::min(units, ctas);
 }
 
