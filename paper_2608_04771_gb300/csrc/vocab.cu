@@ -166,7 +166,8 @@ __device__ __forceinline__ float block_scan_excl(float x, float *sm_w)
 // T among positive values, with the running sum before it; -1 if none (T at or above
 // the total, or NaN).  `last` receives the last index with a positive value (-1: none).
 // A thread whose run the block scan says holds the crossing takes its last positive
-// value when its own sequential sum falls a rounding short of T.
+// value, with the running sum before that value, when its own sequential sum falls a
+// rounding short of T (so the search inside a chosen segment then ends at its top).
 template <int NT, int R>
 __device__ __forceinline__ int find_crossing(const float (&v)[R], int first, float T, float *sm_w, int *sm_i,
                                              float *sm_f, float &before, int &last)
@@ -186,16 +187,18 @@ __device__ __forceinline__ int find_crossing(const float (&v)[R], int first, flo
     }
     __syncthreads();
     if (run > 0.f && excl <= T && excl + run > T) {  // at most one thread: the prefix only grows
-        float c = excl, prev = excl + run;  // defaults: the crossing lost to rounding
+        float c = excl, prev = excl;  // defaults: the crossing lost to rounding
         int pick = my_last;
         bool hit = false;
 #pragma unroll
         for (int k = 0; k < R; ++k) {
             const float c0 = c;
             c += v[k];
-            if (!hit && v[k] > 0.f && c > T) {
-                hit = true;
-                pick = first + k;
+            if (!hit && v[k] > 0.f) {
+                if (c > T) {
+                    hit = true;
+                    pick = first + k;
+                }
                 prev = c0;
             }
         }
