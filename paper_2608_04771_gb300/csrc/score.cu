@@ -176,17 +176,14 @@ __global__ void __launch_bounds__(1024) score_unit_list(const int32_t *__restric
 // mask gives the row, so the decode's natural-log normaliser lse of that query head is
 // the row's: b_r = lse * log2(e).  row_lse is [w][rows_q] (rows_q = layers * B * H_q,
 // query heads in q order).  A non-finite normaliser raises ERR_NORM and leaves the row's
-// normaliser at +inf, so the row adds nothing to the scores.
+// normaliser at +inf, so the row adds nothing to the scores.  The tensor-core pass 2
+// computes the same b_r itself where it loads a row's normaliser; this kernel serves
+// the SIMT pass.
 __global__ void score_rowb_from_lse(const int32_t *__restrict__ lens, ScoreMask mask, int w, int L_cap, int R, int G,
                                     int Hq, int Hkv, long rows_q, const float *__restrict__ row_lse,
-                                    float *__restrict__ rowb, long units, int32_t *__restrict__ ulist,
-                                    int32_t *__restrict__ ucount, unsigned *err)
+                                    float *__restrict__ rowb, long units, unsigned *err)
 {
     wait_prior_grid();  // lens and the ring rows may come from the previous kernels
-    if (ulist != nullptr && blockIdx.x == gridDim.x - 1) {  // the extra block: the units a masked call scores
-        unit_list_block(lens, mask, w, L_cap, (int)units, ulist, ucount);
-        return;
-    }
     const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= units * R) return;
     const long u = i / R;
@@ -363,8 +360,11 @@ __global__ void score_pool(const float *__restrict__ raw, const int32_t *__restr
 
 cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
                                   float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+// row_lse (or nullptr: ws.rowb) gives pass 2 its row normalisers: the decode's lse, read
+// where each row's normaliser is loaded.
 cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
-                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used);
+                                  float c2, const ScoreWs &ws, const float *row_lse, unsigned *err, cudaStream_t s,
+                                  bool *used);
 bool score_tc_supported(const reco_kv &kv, int w);
 int score_tc_pass1_groups(int R);
 
@@ -466,7 +466,7 @@ cudaError_t launch_score(const reco_kv &kv, const void *q_win, const int32_t *le
                 lens, mask, w, kv.L_cap, R, nch, score_tc_pass1_groups(R), ws.part_m, ws.part_z, ws.rowb, units);
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
             bool used2 = false;
-            e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used2);
+            e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, nullptr, err, s, &used2);
             if (e != cudaSuccess) return e;
             if (!used2) return cudaErrorNotSupported;
         }
@@ -537,19 +537,20 @@ cudaError_t launch_score_lse(const reco_kv &kv, const void *q_win, const int32_t
     const long rows_q = (long)kv.n_layers * kv.B * kv.H_q;
     const bool tc = kv.dtype == RECO_BF16 && score_tc_supported(kv, w);
     cudaError_t e;
-    // the row normalisers, and (a masked tensor-core call) the unit list from one extra block
-    const bool listed = tc && keep;
-    const unsigned blocks = (unsigned)((units * R + 255) / 256) + (listed ? 1u : 0u);
-    e = launch_pdl(score_rowb_from_lse, dim3(blocks), dim3(256), 0, s, lens, mask, w, kv.L_cap, R, G, kv.H_q, kv.H_kv,
-                   rows_q, row_lse, ws.rowb, units, listed ? ws.ulist : nullptr, listed ? ws.ucount : nullptr, err);
-    if (e != cudaSuccess) return e;
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     bool used = false;
-    if (tc) {
-        e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, err, s, &used);
+    if (tc) {  // the tensor-core pass reads each row's normaliser from row_lse itself
+        if (keep) {
+            e = launch_pdl(score_unit_list, dim3(1), dim3(1024), 0, s, lens, mask, w, kv.L_cap, (int)units, ws.ulist,
+                           ws.ucount);
+            if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
+        }
+        e = launch_score_tc_pass2(kv, q_win, lens, keep != nullptr, w, c2, ws, row_lse, err, s, &used);
         if (e != cudaSuccess) return e;
     }
-    if (!used) {
+    if (!used) {  // the SIMT pass takes them from ws.rowb
+        e = launch_pdl(score_rowb_from_lse, dim3((unsigned)((units * R + 255) / 256)), dim3(256), 0, s, lens, mask, w,
+                       kv.L_cap, R, G, kv.H_q, kv.H_kv, rows_q, row_lse, ws.rowb, units, err);
+        if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
         e = score_simt_any(kv, q_win, lens, mask, w, c2, ws, err, s, false);
         if (e != cudaSuccess) return e;
     }

@@ -521,7 +521,7 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                     const int32_t *__restrict__ lens, int w, int G, int Hq, int Hkv, int L_cap, int R, int NQ, int NP,
                     int NR, int NS, int n_chunks, int n_items, const int32_t *__restrict__ ulist,
                     const int32_t *__restrict__ ucount, float c2, const float *__restrict__ rowb,
-                    float *__restrict__ raw, unsigned *err)
+                    const float *__restrict__ row_lse, long rows_q, float *__restrict__ raw, unsigned *err)
 {
     constexpr int HALVES = D / 64;
     constexpr int KBOX = 128 * 128;  // 128 keys x 128 bytes
@@ -695,7 +695,21 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                 __syncwarp();          // +inf for padding columns, which then add exp2(-inf) = 0
                 for (int q = lane; q < NP * 64; q += 32) {
                     const int h = q >> 6, c = q & 63, rr = h * NW + c_lo + c;
-                    bs[q] = (c < nc && rr < R) ? rowb[it.u * R + rr] : INFINITY;
+                    float b = INFINITY;
+                    if (c < nc && rr < R) {
+                        if (row_lse != nullptr) {  // row (g, t) of the window: the decode's lse of that query
+                            const long qi = (it.u / Hkv) * Hq + (it.u % Hkv) * G + rr / w;
+                            const float l = row_lse[(long)(rr % w) * rows_q + qi];
+                            if (isfinite(l)) {
+                                b = l * kLog2e;
+                            } else {  // the row adds nothing; the device error word says why
+                                raise_error(err, ERR_NORM);
+                            }
+                        } else {
+                            b = rowb[it.u * R + rr];
+                        }
+                    }
+                    bs[q] = b;
                 }
                 __syncwarp();
                 prev_u = it.u;
@@ -824,7 +838,8 @@ cudaError_t launch_score_tc_pass1(const reco_kv &kv, const void *q_win, const in
 
 template <int D>
 static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
-                             float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
+                             float c2, const ScoreWs &ws, const float *row_lse, unsigned *err, cudaStream_t s,
+                             bool *ok)
 {
     const long units = (long)kv.n_layers * kv.B * kv.H_kv;
     const int R = (kv.H_q / kv.H_kv) * w;
@@ -853,18 +868,20 @@ static cudaError_t run_pass2(const reco_kv &kv, const void *q_win, const int32_t
     const int grid = min(n_items, device_sm_count());
     e = launch_pdl(score_colsum_tc<D>, dim3(grid), dim3(128 + 128 * kP2Groups), smem, s, mq, mk, lens, w,
                    kv.H_q / kv.H_kv, kv.H_q, kv.H_kv, kv.L_cap, R, ps.NQ, ps.NP, ps.NR, NS, nch, n_items,
-                   masked ? ws.ulist : nullptr, masked ? ws.ucount : nullptr, c2, ws.rowb, ws.raw, err);
+                   masked ? ws.ulist : nullptr, masked ? ws.ucount : nullptr, c2, (const float *)ws.rowb, row_lse,
+                   (long)kv.n_layers * kv.B * kv.H_q, ws.raw, err);
     *ok = true;
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_score_tc_pass2(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
-                                  float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *used)
+                                  float c2, const ScoreWs &ws, const float *row_lse, unsigned *err, cudaStream_t s,
+                                  bool *used)
 {
     *used = false;
     if (!score_tc_supported(kv, w)) return cudaSuccess;
-    return kv.d == 128 ? run_pass2<128>(kv, q_win, lens, masked, w, c2, ws, err, s, used)
-                       : run_pass2<64>(kv, q_win, lens, masked, w, c2, ws, err, s, used);
+    return kv.d == 128 ? run_pass2<128>(kv, q_win, lens, masked, w, c2, ws, row_lse, err, s, used)
+                       : run_pass2<64>(kv, q_win, lens, masked, w, c2, ws, row_lse, err, s, used);
 }
 
 }  // namespace reco
