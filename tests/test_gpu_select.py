@@ -171,3 +171,17 @@ def test_compact_refuses_indices_outside_r_to_L():
         np.testing.assert_array_equal(Kb[0, 1, 0, r], K0b[0, 1, 0, r if src is None else src])
     assert lens.flatten().tolist() == [8, 8]
     reco.reco_check()
+
+
+@pytest.mark.parametrize("split", [False, True])
+def test_select_compact_walks_many_units_with_untouched_sequences(split):
+    """8192 units (64 layers x 16 sequences x 8 KV heads): every CTA walks a few dozen units.
+    Half the sequences keep their whole cache (keep = L: identity indices, nothing moves, the
+    compaction skips them) and the others compress, with ties."""
+    wl = W.WORKLOADS["7b"].reduced(layers=64, batch=16, h_q=8, h_kv=8, L=96, w=8, decode_steps=0)
+    rng = np.random.default_rng(77)
+    L_seq = rng.integers(40, 97, wl.batch)
+    lens_np = np.broadcast_to(L_seq[None, :, None], (wl.layers, wl.batch, wl.h_kv)).astype(np.int32).copy()
+    keep_np = np.where(np.arange(wl.batch) % 2 == 0, L_seq, rng.integers(wl.w, L_seq)).astype(np.int32)
+    scores_np = _tie_scores(rng, (wl.layers, wl.batch, wl.h_kv, wl.L_cap), 16)
+    _run_case(wl, lens_np, keep_np, scores_np, split=split)
