@@ -74,6 +74,8 @@ struct DecodeArgs {
     long long nq;     // query heads of the launch (layers * B * H_q)
     void *qring;      // or nullptr: [nq][slots][D] of q's dtype, row *slot of every head gets its query
     int q_bytes;      // bytes per element of q
+    long long nq_rows;  // query heads of this launch (nq, or a part of it when the units are split)
+    int advance;        // this launch advances *slot (the last of a split launch's parts)
 };
 
 // The ring row this launch writes (read once the previous kernel's writes are visible),
@@ -654,7 +656,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     // are in flight
     if (a.qring != nullptr && rs >= 0) {
         constexpr int CH = D / 8;  // 16-byte chunks of a bf16 query row
-        const long long n16 = a.nq * CH;
+        const long long n16 = a.nq_rows * CH;
         const int tw = (int)gridDim.x * NW, me = (int)blockIdx.x * NW + wid;
         const long long per = (n16 + tw - 1) / tw;
         const long long c0 = min(n16, (long long)me * per), c1 = min(n16, c0 + per);
@@ -1021,7 +1023,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         __syncwarp();
         if (lane == 0) {
             *reinterpret_cast<unsigned long long *>(a.counters) = 0ull;
-            if (rs >= 0) *a.slot = (rs + 1) % a.slots;  // every warp has read the row by now
+            if (rs >= 0 && a.advance) *a.slot = (rs + 1) % a.slots;  // every warp has read the row by now
         }
     }
 }
@@ -1083,26 +1085,53 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
     a.nq = (long long)kv.n_layers * kv.B * kv.H_q;
     a.qring = ring ? qring : nullptr;
     a.q_bytes = kv.dtype == RECO_F32 ? 4 : 2;
-    const unsigned long long rows = (unsigned long long)a.units * kv.L_cap;
+    a.nq_rows = a.nq;
+    a.advance = 1;
     // partial slots: two per warp of the grid
     const bool slots_fit = 2LL * device_sm_count() * kDecodeWarps <= (long long)ws.part_slots;
     // the TMA path takes up to 8 query heads per unit; a unit of G <= 16 heads is two
     // virtual units of ceil(G / 2) heads each
     a.hs = a.G > 8 ? 2 : 1;
     a.gv = (a.G + a.hs - 1) / a.hs;
-    if (kv.dtype == RECO_BF16 && a.G <= 16 && (long long)a.units * a.hs <= kMaxTmaUnits && rows < (1ull << 31) &&
-        slots_fit) {
-        DecodeArgs at = a;  // virtual units
-        at.units *= at.hs;
-        CUtensorMap mk, mv;
-        if (encode_cache_map(&mk, kv.k, rows, kv.d) && encode_cache_map(&mv, kv.v, rows, kv.d)) {
+    // More units than one plan holds in shared memory run as consecutive launches over
+    // contiguous unit ranges (every unit is independent): each part gets its own K/V, q,
+    // output, lens and ring pointers, and only the last part advances the ring slot.
+    const long long part_units = kMaxTmaUnits / a.hs;  // cache units per launch
+    if (kv.dtype == RECO_BF16 && a.G <= 16 && (unsigned long long)std::min<long long>(a.units, part_units) * kv.L_cap <
+                                                   (1ull << 31) && slots_fit) {
+        const bool two = a.hs == 2;
+        const void *fn = kv.d == 64 ? (two ? (const void *)decode_tma<64, 2> : (const void *)decode_tma<64, 1>)
+                                    : (two ? (const void *)decode_tma<128, 2> : (const void *)decode_tma<128, 1>);
+        const size_t row_b = (size_t)kv.d * 2;  // bf16 cache and query rows
+        const size_t out_b = (size_t)kv.d * (out_dtype == RECO_BF16 ? 2 : 4);
+        for (long long u0 = 0; u0 < a.units; u0 += part_units) {
+            const long long cu = std::min(part_units, (long long)a.units - u0);
+            const long long q0 = u0 * a.G;  // first query head of the part
+            const unsigned long long rows = (unsigned long long)cu * kv.L_cap;
+            CUtensorMap mk, mv;
+            const char *kb = static_cast<const char *>(kv.k) + (size_t)u0 * kv.L_cap * row_b;
+            const char *vb = static_cast<const char *>(kv.v) + (size_t)u0 * kv.L_cap * row_b;
+            if (!encode_cache_map(&mk, kb, rows, kv.d) || !encode_cache_map(&mv, vb, rows, kv.d)) {
+                if (u0 == 0) break;  // the SIMT path below takes the whole call
+                return cudaErrorInvalidValue;
+            }
+            DecodeArgs at = a;  // virtual units of this part
+            at.units = (int)(cu * a.hs);
+            at.K = const_cast<char *>(kb);
+            at.V = const_cast<char *>(vb);
+            at.q = static_cast<const char *>(q) + (size_t)q0 * row_b;
+            at.k_new = k_new ? static_cast<const char *>(k_new) + (size_t)u0 * row_b : nullptr;
+            at.v_new = v_new ? static_cast<const char *>(v_new) + (size_t)u0 * row_b : nullptr;
+            at.lens = lens + u0;
+            at.out = static_cast<char *>(out) + (size_t)q0 * out_b;
+            at.lse = lse ? lse + q0 : nullptr;
+            at.ring = ring ? ring + q0 : nullptr;  // ring rows keep their full stride nq
+            at.qring = a.qring ? static_cast<char *>(a.qring) + (size_t)q0 * slots * row_b : nullptr;
+            at.nq_rows = cu * a.G;
+            at.advance = u0 + cu >= a.units ? 1 : 0;
             // the counters are zero on entry (zero-filled workspace) and every launch leaves them so
-            cudaError_t e;
             const size_t smem = kv.d == 64 ? tma_smem_bytes<64>(at.units) : tma_smem_bytes<128>(at.units);
-            const bool two = at.hs == 2;
-            const void *fn = kv.d == 64 ? (two ? (const void *)decode_tma<64, 2> : (const void *)decode_tma<64, 1>)
-                                        : (two ? (const void *)decode_tma<128, 2> : (const void *)decode_tma<128, 1>);
-            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
             const int grid = device_sm_count();
             const dim3 blk(kDecodeWarps * 32);
@@ -1112,7 +1141,8 @@ cudaError_t launch_decode(const reco_kv &kv, const void *q, const void *k_new, c
             else
                 e = two ? launch_pdl(decode_tma<128, 2>, dim3(grid), blk, smem, s, mk, mv, at)
                         : launch_pdl(decode_tma<128, 1>, dim3(grid), blk, smem, s, mk, mv, at);
-            return e != cudaSuccess ? e : cudaGetLastError();
+            if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
+            if (u0 + cu >= a.units) return cudaSuccess;
         }
     }
     a.hs = 1;

@@ -153,14 +153,15 @@ def test_deep_ring_partition_ragged():
     _check(wl, lens, True, steps=2)
 
 
-@pytest.mark.parametrize("shape", [(64, 16, 56, 8), (1, 8193, 7, 1)])
+@pytest.mark.parametrize("shape", [(64, 16, 56, 8), (1, 8193, 7, 1), (2, 4100, 8, 1), (1, 4097, 16, 1)])
 def test_tma_path_unit_limit(shape):
-    """8192 units (the most the TMA path plans in shared memory) and 8193 (the SIMT path)."""
+    """8192 units (the most one TMA launch plans in shared memory), then more: 8193 and 8200
+    units run as two launches over unit ranges, and so do 4097 units of 16 heads (two
+    virtual units each)."""
     layers, batch, h_q, h_kv = shape
     wl = W.WORKLOADS["7b"].reduced(layers=layers, batch=batch, h_q=h_q, h_kv=h_kv, L=40, decode_steps=4)
     rng = np.random.default_rng(42 + layers)
     lens = rng.integers(1, 41, (layers, batch, h_kv)).astype(np.int32)
-    assert lens.size in (8192, 8193)
     _check(wl, lens, True)
 
 

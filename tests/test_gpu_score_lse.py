@@ -271,3 +271,33 @@ def test_copy_row_selects_the_row_on_the_device():
         assert e.value.status == reco.RECO_EDEVICE
         assert torch.equal(dst, before)
     reco.reco_check()
+
+
+def test_decode_attn_ring_split_over_unit_ranges():
+    """8200 units run as two launches: the lse of every query head in ring rows slot and
+    slot + S, its query in q_ring row slot, the outputs and lengths those of reco_decode_attn,
+    and the slot advanced once."""
+    wl = W.WORKLOADS["7b"].reduced(layers=2, batch=1025, h_q=28, h_kv=4, L=48, decode_steps=2)
+    assert wl.layers * wl.batch * wl.h_kv > 8192
+    Ka, Va = W.make_cache(wl, DEV, canary=False)
+    Kb, Vb = Ka.clone(), Va.clone()
+    rng = np.random.default_rng(9)
+    lens_np = rng.integers(1, 40, (wl.layers, wl.batch, wl.h_kv)).astype(np.int32)
+    la, lb = torch.from_numpy(lens_np).to(DEV), torch.from_numpy(lens_np).to(DEV)
+    kva, kvb = reco.make_kv(Ka, Va, wl.h_q), reco.make_kv(Kb, Vb, wl.h_q)
+    wsa, wsb = reco.workspace(reco.RECO_OP_DECODE, kva, 0, DEV), reco.workspace(reco.RECO_OP_DECODE, kvb, 0, DEV)
+    S, n = 2, wl.layers * wl.batch * wl.h_q
+    ring = torch.zeros((2 * S, n), device=DEV)
+    slot = torch.tensor([1], dtype=torch.int64, device=DEV)
+    q_ring = torch.zeros((wl.layers, wl.batch, wl.h_q, S, wl.d), dtype=wl.torch_dtype, device=DEV)
+    q, kn, vn = W.make_decode_step(wl, 0, DEV)
+    oa, ob = torch.empty(q.shape, device=DEV), torch.empty(q.shape, device=DEV)
+    lse = torch.empty(q.shape[:3], device=DEV)
+    reco.reco_decode_attn(kva, q, kn, vn, la, wl.scale(), oa, lse, wsa)
+    reco.reco_decode_attn_ring(kvb, q, kn, vn, lb, wl.scale(), ob, ring, slot, wsb, q_ring=q_ring)
+    reco.reco_check()
+    assert torch.equal(oa, ob) and torch.equal(la, lb) and int(slot.item()) == 0
+    assert torch.equal(ring[1], lse.view(-1)) and torch.equal(ring[1 + S], lse.view(-1))
+    assert torch.equal(ring[0], torch.zeros_like(ring[0])) and torch.equal(ring[S], torch.zeros_like(ring[0]))
+    assert torch.equal(q_ring[:, :, :, 1], q) and torch.equal(q_ring[:, :, :, 0], torch.zeros_like(q))
+    assert torch.equal(Ka.view(torch.uint8), Kb.view(torch.uint8))
