@@ -139,6 +139,14 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def decode_code_hash(src: str) -> str:
+    """sha256 (16 hex digits) of a CUDA source with its comments and blank lines removed:
+    a profile stays valid across edits that change no code."""
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    lines = [re.sub(r"//.*$", "", ln).rstrip() for ln in src.splitlines()]
+    return hashlib.sha256("\n".join(ln for ln in lines if ln.strip()).encode()).hexdigest()[:16]
+
+
 def decode_traffic(wl):
     """DRAM bytes per decode launch of this workload from the committed ncu summary
     profiles/decode_attn_<workload>.md, if it was taken on the current decode kernel
@@ -153,8 +161,8 @@ def decode_traffic(wl):
     c = re.search(r"capture:\s*(.+)", text)
     if not m or not h:
         return None, f"none: profiles/{name} carries no per-launch DRAM bytes"
-    src = open(os.path.join(ROOT, "paper_2608_04771_gb300", "csrc", "decode.cu"), "rb").read()
-    if hashlib.sha256(src).hexdigest()[:16] != h.group(1)[:16]:
+    src = open(os.path.join(ROOT, "paper_2608_04771_gb300", "csrc", "decode.cu")).read()
+    if decode_code_hash(src) != h.group(1)[:16]:
         return None, f"none: profiles/{name} was taken on another decode.cu"
     return float(m.group(1)), (f"profile-derived, not measured in this run: profiles/{name} "
                                f"(ncu dram__bytes_read.sum + dram__bytes_write.sum; {c.group(1).strip() if c else ''})")

@@ -2,9 +2,11 @@
 // attention whose cost the compression lowers (Sec. 1; Sec. 2.2; Sec. 4.2).
 //
 // bf16 path (decode_tma): a persistent split-K flash-decode, one CTA of 8 warps per
-// SM (for long work 4 of them, each with a ring twice as deep).  Every CTA first builds the same work plan from lens: the prefix sum of 16-key
-// blocks per unit, with the blocks of all units laid end to end and cut into one equal
-// contiguous range per warp (a stream-K split: balanced to one block, no work queue).
+// SM (for long work 4 of them, each with a ring twice as deep).  Every CTA first
+// builds the same work plan from lens: the prefix sum of 16-key blocks per unit, with
+// the blocks of all units laid end to end and cut into one equal contiguous range per
+// warp (a stream-K split: balanced to one block, no work queue).  A call with more units
+// than one plan holds runs as consecutive launches over contiguous unit ranges.
 // When no unit is long enough to be cut, the units are instead sorted by length and
 // dealt whole to the warps in snake order (longest first).
 // An item's keys stream from HBM in 16-key blocks: one lane issues TMA tensor copies
@@ -13,12 +15,13 @@
 // m16n8k16 (bf16 in, fp32 accumulate) with the G <= 8 query heads of the KV head
 // packed into one MMA tile.  The head dimension is permuted consistently on the Q
 // and K sides (and on the V and output sides) so that each thread's fragments are
-// whole 16-byte chunks, and the swizzle makes every fragment read conflict-free.  A unit split over several items writes partial
-// (max, sum, output) triples; the last item to finish (atomic ticket, no waiting)
-// merges them.  The counters live in the caller's workspace, zero-filled before its
-// first use; each launch clears what it counted, so no reset runs between launches.  The appended token (k_new, v_new) is read from the inputs and written
-// into the cache by the warp that covers its index; the last warp of the grid to
-// finish advances lens.
+// whole 16-byte chunks, and the swizzle makes every fragment read conflict-free.  A
+// unit split over several items writes partial (max, sum, output) triples; the last
+// item to finish (atomic ticket, no waiting) merges them.  The counters live in the
+// caller's workspace, zero-filled before its first use; each launch clears what it
+// counted, so no reset runs between launches.  The appended token (k_new, v_new) is
+// read from the inputs and written into the cache by the warp that covers its index;
+// the last warp of the grid to finish advances lens.
 //
 // float32 path (decode_simt): one CTA per unit, four warps over the keys, G <= 16.
 #include <cuda.h>
