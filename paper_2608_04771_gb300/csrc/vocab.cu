@@ -537,17 +537,10 @@ cudaError_t launch_penalty_sample(float *logits, int B, int V, const int32_t *id
                       (const float2 *)part, tokens);
 }
 
-// Online (max, sum) in the log2 domain over four values.
-__device__ __forceinline__ void ms_add4(float &m, float &s, float a, float b, float c, float d)
-{
-    const float mx = fmaxf(fmaxf(a, b), fmaxf(c, d));
-    if (mx > m) {
-        s *= fast_exp2(m - mx);
-        m = mx;
-    }
-    s += fast_exp2(a - m) + fast_exp2(b - m) + fast_exp2(c - m) + fast_exp2(d - m);
-}
-
+// One row's Eq. 5 term per CTA: one streaming pass over the row's logits for their
+// log2-domain (max, sum), then lp = z[x] - logsumexp(z).  (Four CTAs per row in a cluster,
+// merged through CTA 0's shared memory, measured slower: 38.9 against 31.1 us at 8 x 32 rows
+// of 152064 logits.)
 template <int NT>
 __global__ void __launch_bounds__(NT) ppl_rows(const float *__restrict__ logits,
                                                const int32_t *__restrict__ tokens,
@@ -555,6 +548,7 @@ __global__ void __launch_bounds__(NT) ppl_rows(const float *__restrict__ logits,
                                                float *__restrict__ lp, unsigned *err)
 {
     __shared__ float sm_m[NT / 32], sm_s[NT / 32];
+    wait_prior_grid();  // the logits may come from the previous kernel
     const int t = blockIdx.x, b = blockIdx.y;
     const int nb = n_valid ? min(n_valid[b], n) : n;
     if (t >= nb) return;
@@ -563,10 +557,31 @@ __global__ void __launch_bounds__(NT) ppl_rows(const float *__restrict__ logits,
     // Vector loads only when every row starts on a 16-byte boundary: the base is
     // 16-byte aligned and rows are a multiple of 4 floats long.
     if ((V & 3) == 0 && ((uintptr_t)logits & 15u) == 0) {
+        // eight 16-byte loads per thread in flight, then one max and 32 exponentials
         const float4 *z4 = reinterpret_cast<const float4 *>(z);
-        for (int i = threadIdx.x; i < V / 4; i += NT) {
-            const float4 x = __ldcs(z4 + i);
-            ms_add4(m, s, x.x * kLog2e, x.y * kLog2e, x.z * kLog2e, x.w * kLog2e);
+        const int n4 = V / 4;
+        constexpr float NINF = -INFINITY;
+        for (int i0 = threadIdx.x; i0 < n4; i0 += 8 * NT) {
+            float4 x[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int i = i0 + k * NT;
+                x[k] = i < n4 ? __ldcs(z4 + i) : make_float4(NINF, NINF, NINF, NINF);
+            }
+            float mx = NINF;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) mx = fmaxf(mx, fmaxf(fmaxf(x[k].x, x[k].y), fmaxf(x[k].z, x[k].w)));
+            mx *= kLog2e;
+            if (mx > m) {
+                s *= fast_exp2(m - mx);  // m = -inf: s is 0 and stays 0
+                m = mx;
+            }
+            if (m != NINF) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    s += (fast_exp2(fmaf(x[k].x, kLog2e, -m)) + fast_exp2(fmaf(x[k].y, kLog2e, -m))) +
+                         (fast_exp2(fmaf(x[k].z, kLog2e, -m)) + fast_exp2(fmaf(x[k].w, kLog2e, -m)));
+            }
         }
     } else {
         for (int i = threadIdx.x; i < V; i += NT) {
@@ -594,20 +609,21 @@ __global__ void __launch_bounds__(NT) ppl_rows(const float *__restrict__ logits,
         float M = sm_m[0], S = sm_s[0];
         for (int w2 = 1; w2 < NT / 32; ++w2) lse_merge(M, S, sm_m[w2], sm_s[w2]);
         const int x = tokens[(size_t)b * n + t];
-        float r;
+        float res;
         if (x < 0 || x >= V) {
             raise_error(err, ERR_TOKEN);
-            r = __int_as_float(0x7fc00000);
+            res = __int_as_float(0x7fc00000);
         } else {
-            r = z[x] - (M + log2f(S)) * kLn2;
+            res = z[x] - (M + log2f(S)) * kLn2;
         }
-        lp[(size_t)b * n + t] = r;
+        lp[(size_t)b * n + t] = res;
     }
 }
 
 __global__ void ppl_finish(const float *__restrict__ lp, const int32_t *__restrict__ n_valid, int B, int n,
                            float tau_p, float *__restrict__ ppl, uint8_t *__restrict__ stop)
 {
+    wait_prior_grid();  // the row terms come from ppl_rows
     const int b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= B) return;
     const int nb = n_valid ? min(n_valid[b], n) : n;
@@ -627,13 +643,13 @@ cudaError_t launch_ppl(const float *logits, const int32_t *tokens, const int32_t
                        int V, float tau_p, float *ppl, uint8_t *stop, float *lp_ws, unsigned *err,
                        cudaStream_t s)
 {
+    cudaError_t e;
     if (n > 0) {
-        ppl_rows<512><<<dim3(n, B), 512, 0, s>>>(logits, tokens, n_valid, n, V, lp_ws, err);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+        e = launch_pdl(ppl_rows<512>, dim3(n, B), dim3(512), 0, s, logits, tokens, n_valid, n, V, lp_ws, err);
+        if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    ppl_finish<<<(B + 127) / 128, 128, 0, s>>>(lp_ws, n_valid, B, n, tau_p, ppl, stop);
-    return cudaGetLastError();
+    e = launch_pdl(ppl_finish, dim3((B + 127) / 128), dim3(128), 0, s, lp_ws, n_valid, B, n, tau_p, ppl, stop);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace reco
