@@ -580,7 +580,7 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
     if (warp == 0) {
         if (lane == 0) {  // producer
             const int qbox_rows = NQ > 256 ? NQ / 2 : NQ;
-            int gt = 0, nq = 0;
+            int s = 0, kph = 0, nq = 0;  // K stage and the parity of its round
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
@@ -598,9 +598,8 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                     prev_u = it.u;
                 }
                 const int k_row0 = (int)(it.u * L_cap + it.j0);
-                for (int t = 0; t < it.ntiles; ++t, ++gt) {
-                    const int s = gt % NS;
-                    if (!wait_or_flag(smem_addr(&bar_kempty[s]), ((gt / NS) & 1) ^ 1, abort_flag, err)) {
+                for (int t = 0; t < it.ntiles; ++t) {
+                    if (!wait_or_flag(smem_addr(&bar_kempty[s]), kph ^ 1, abort_flag, err)) {
                         ok = false;
                         break;
                     }
@@ -608,13 +607,17 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                     for (int hh = 0; hh < HALVES; ++hh)
                         tma_load_2d(Ks + s * KSTAGE + hh * KBOX, &tmK, 64 * hh, k_row0 + t * 128,
                                     smem_addr(&bar_kfull[s]));
+                    if (++s == NS) {
+                        s = 0;
+                        kph ^= 1;
+                    }
                 }
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {  // MMA issuer: one chain per piece
             const uint32_t idesc = idesc_bf16(128, NW);
-            int gt = 0, nq = 0;
+            int s = 0, kph = 0, b = 0, aph = 0, nq = 0;  // K stage, accumulator region, their parities
             long prev_u = -1;
             bool ok = true;
             for (int i = i_begin; ok && i < i_end; ++i) {
@@ -626,15 +629,13 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                     ++nq;
                     prev_u = it.u;
                 }
-                for (int t = 0; ok && t < it.ntiles; ++t, ++gt) {
-                    const int s = gt % NS;
-                    if (!wait_or_flag(smem_addr(&bar_kfull[s]), (gt / NS) & 1, abort_flag, err)) {
+                for (int t = 0; ok && t < it.ntiles; ++t) {
+                    if (!wait_or_flag(smem_addr(&bar_kfull[s]), kph, abort_flag, err)) {
                         ok = false;
                         break;
                     }
                     for (int h = 0; h < NP; ++h) {
-                        const int p = gt * NP + h, b = p % NR;
-                        if (!wait_or_flag(smem_addr(&bar_aempty[b]), ((p / NR) & 1) ^ 1, abort_flag, err)) {
+                        if (!wait_or_flag(smem_addr(&bar_aempty[b]), aph ^ 1, abort_flag, err)) {
                             ok = false;
                             break;
                         }
@@ -651,8 +652,16 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                                    idesc, k > 0 ? 1u : 0u);
                         }
                         tc_commit(smem_addr(&bar_afull[b]));
+                        if (++b == NR) {
+                            b = 0;
+                            aph ^= 1;
+                        }
                     }
                     if (ok) tc_commit(smem_addr(&bar_kempty[s]));
+                    if (++s == NS) {
+                        s = 0;
+                        kph ^= 1;
+                    }
                 }
             }
         }
@@ -685,7 +694,7 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
         const int row = quarter * 32 + lane;  // key within the tile
         const int c_lo = split8_lo(NW, EG, g), nc = split8_lo(NW, EG, g + 1) - c_lo;
         float *bs = bsh[warp - 4];
-        int gt = 0;
+        int gt = 0, b = 0, aph = 0;  // tile count; accumulator region and its parity
         long prev_u = -1;
         bool ok = true;
         for (int i = i_begin; ok && i < i_end; ++i) {
@@ -717,8 +726,7 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
             for (int t = 0; t < it.ntiles; ++t, ++gt) {
                 float a4[4] = {0.f, 0.f, 0.f, 0.f};
                 for (int h = 0; h < NP; ++h) {
-                    const int p = gt * NP + h, b = p % NR;
-                    if (!wait_or_flag(smem_addr(&bar_afull[b]), (p / NR) & 1, abort_flag, err)) {
+                    if (!wait_or_flag(smem_addr(&bar_afull[b]), aph, abort_flag, err)) {
                         ok = false;
                         break;
                     }
@@ -737,6 +745,10 @@ __global__ void __launch_bounds__(128 + 128 * kP2Groups, 1)
                         tmem_ld_wait_regs<32>(v[1]);
                         colsum_release(lane, bar_aempty[b]);
                         colsum_batch(v[1], n1, bh + 32, c2, a4);
+                    }
+                    if (++b == NR) {
+                        b = 0;
+                        aph ^= 1;
                     }
                 }
                 if (!ok) break;
