@@ -15,8 +15,8 @@
 // while the epilogue groups work on earlier ones.
 //
 // Pass 1 (row statistics): queries on M (128-row tiles), keys on N, so each thread owns
-//   one window row and keeps a running (reference, sum) over the chunk's keys.  Two
-//   epilogue groups take alternate key tiles and leave one partial each.  A full tile
+//   one window row and keeps a running (reference, sum) over the chunk's keys.  The
+//   epilogue groups split each tile's key columns and leave one partial each.  A full tile
 //   is exponentiated against the row's current reference without a max pass; only a
 //   row's first tile, a masked tile, or a tile whose sum could overflow takes its max.
 // Pass 2 (column sums): keys on M (128 per tile), queries on N, split into up to four
@@ -826,6 +826,10 @@ static cudaError_t run_pass1(const reco_kv &kv, const void *q_win, const int32_t
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// Key tiles of 256 for two query tiles: half the MMA instructions per key of 128-key tiles
+// (the single issuing thread is the pass's bottleneck; 7B-class heads, both passes 2.03 ->
+// 1.85 ms), with two 256-column TMEM regions and two K stages in shared memory.  Three or
+// four query tiles leave shared memory for one such stage only and keep 128-key tiles.
 template <int D>
 static cudaError_t pass1_by_mt(const reco_kv &kv, const void *q_win, const int32_t *lens, bool masked, int w,
                                float c2, const ScoreWs &ws, unsigned *err, cudaStream_t s, bool *ok)
@@ -833,7 +837,7 @@ static cudaError_t pass1_by_mt(const reco_kv &kv, const void *q_win, const int32
     const int MT = ((kv.H_q / kv.H_kv) * w + 127) / 128;
     switch (MT) {
     case 1: return run_pass1<D, 1, 128, 2>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
-    case 2: return run_pass1<D, 2, 128, 2>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
+    case 2: return run_pass1<D, 2, 256, 2>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);  // 256-key tiles
     case 3: return run_pass1<D, 3, 128, 2>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
     default: return run_pass1<D, 4, 128, 1>(kv, q_win, lens, masked, w, c2, ws, err, s, ok);
     }
