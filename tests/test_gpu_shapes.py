@@ -24,6 +24,8 @@ CASES = {
     # name: overrides                                       path exercised
     "mha_g1": dict(h_q=4, h_kv=4, w=16, L=900),            # G = 1
     "g3_d64_pool3": dict(h_q=6, h_kv=2, w=8, d=64, pool=3, L=700),
+    "g4_d64_r160": dict(h_q=8, h_kv=2, w=40, d=64, L=1100),  # 2 query tiles at d = 64: pass 1 on 256-key tiles
+    "g7_short_units": dict(L=200),                           # 2 query tiles, every unit inside one 256-key tile
     "g8_r256": dict(h_q=16, h_kv=2, w=32, L=1300),         # tensor decode at G = 8; pass 2 N = 256
     "g16_split_decode": dict(h_q=16, h_kv=1, w=16, L=800),  # G = 16: the TMA decode as two 8-head units
     "w1_pool1": dict(w=1, pool=1, L=600),                  # one window query, Eq. 2 without pooling
